@@ -1,0 +1,251 @@
+"""fp64 CPU oracle for streaming frame-chunk attention over a rolling KV cache.
+
+TEST INFRASTRUCTURE. Only ``tests/``, ``__graft_entry__.smoke()`` and the
+CPU-baseline / reference legs of ``bench.py`` may import this module. The
+product path (``paper_2607_18171_gb300``) never imports it, and this module
+imports nothing from the product path: the two share no arithmetic.
+
+What it computes, and where that comes from
+-------------------------------------------
+The paper (arxiv 2607.18171, "FlashRT") models an autoregressive video DiT
+as an operation whose batch ``j`` inherits a persistent KV cache from batch
+``j-1`` (section 2, "Problem Formulation": the lambda=1 cross-batch state
+edge; Appendix A.1.2 "Pipeline graph": the KV cache shared by batch j+1 and
+batch j), with each denoising step owning an independent cache (section 3.1
+"Case study"; Appendix A.4). Input arrives as frame chunks (Appendix A.1.1).
+The paper gives no formula for the attention itself; the per-chunk
+computation below is the plain definition of the workload the paper's video
+world models run (sections 4.3.2-4.3.4): 3D rotary position embedding on
+Q and K, append of the chunk's K/V to a sliding-window cache, and exact
+softmax attention of the chunk's queries over every cached key.
+
+Every function is the plain definition: no online softmax, no tiling, no
+fused steps. Library primitives used as steps: ``numpy.matmul`` (dot
+products), ``numpy.exp``, ``numpy.cos``/``numpy.sin``.
+
+Readings of points the paper leaves open (each is a convention choice):
+  * RoPE pairs are adjacent elements (2j, 2j+1) inside each of the three
+    head_dim segments [t | h | w]; pair j of a segment of width d_a turns by
+    pos_a * theta**(-2j/d_a), theta = 10000.
+  * Positions: t = chunk * frames_per_chunk + frame (absolute frame index
+    since stream start), (h, w) = row-major place inside the frame.
+  * The window W counts the current chunk: after appending chunk c the cache
+    holds chunks max(0, c-W+1) .. c, and chunk c-W is evicted.
+  * Every query of the chunk attends every cached key (bidirectional inside
+    the chunk, all earlier chunks of the window).
+  * Rotated Q and K are rounded to bf16 before attention (they are stored in
+    bf16); ``exact=True`` keeps them in fp64 for diagnostics.
+"""
+
+from __future__ import annotations
+
+import collections
+import math
+
+import numpy as np
+
+__all__ = [
+    "bf16_round",
+    "token_positions",
+    "rope_angles",
+    "rope3d",
+    "attention",
+    "window_index",
+    "OracleStream",
+]
+
+
+# ---------------------------------------------------------------------------
+# bf16 rounding (IEEE-style round to nearest, ties to even, 8-bit significand)
+# ---------------------------------------------------------------------------
+def bf16_round(x) -> np.ndarray:
+    """Round float64 values to the nearest bfloat16 value (ties to even).
+
+    bfloat16 keeps 8 significant bits (1 implicit + 7 stored) and the float32
+    exponent range. For |x| in [2**E, 2**(E+1)) the spacing is 2**(E-7);
+    below the smallest normal (2**-126) the spacing stays 2**-133. Values that
+    round past the largest finite bf16 become +-inf. The result is returned
+    as float64 (every bf16 value is exact in float64).
+    """
+    x = np.asarray(x, dtype=np.float64)
+    out = x.copy()
+    nz = np.isfinite(x) & (x != 0.0)
+    if not np.any(nz):
+        return out
+    xv = x[nz]
+    _, e = np.frexp(xv)  # xv = m * 2**e, 0.5 <= |m| < 1  ->  leading bit 2**(e-1)
+    lead = np.maximum(e - 1, -126)
+    ulp = np.ldexp(1.0, lead - 7)
+    r = np.rint(xv / ulp) * ulp  # rint: round half to even
+    r = np.where(np.abs(r) >= 2.0**128, np.copysign(np.inf, xv), r)
+    out[nz] = r
+    return out
+
+
+# ---------------------------------------------------------------------------
+# 3D rotary position embedding
+# ---------------------------------------------------------------------------
+def token_positions(chunk: int, n_tokens: int, grid_h: int, grid_w: int):
+    """(t, h, w) position of every token of ``chunk`` (frame-chunk input of
+    Appendix A.1.1). Token i of the chunk is frame f = i // (grid_h*grid_w),
+    row r = (i mod grid_h*grid_w) // grid_w, column i mod grid_w. The returned
+    t is the within-chunk frame f; the caller adds chunk * frames_per_chunk.
+    """
+    tpf = grid_h * grid_w
+    i = np.arange(n_tokens, dtype=np.int64)
+    f = i // tpf
+    r = (i % tpf) // grid_w
+    col = i % grid_w
+    return f, r, col
+
+
+def rope_angles(pos: np.ndarray, width: int, theta: float) -> np.ndarray:
+    """Angle of pair j at integer position ``pos`` in a segment of ``width``
+    dims: pos * theta**(-2j/width), j = 0 .. width/2 - 1. Shape [len(pos), width/2]."""
+    j = np.arange(width // 2, dtype=np.float64)
+    inv_freq = np.power(float(theta), -2.0 * j / float(width))
+    return np.outer(np.asarray(pos, dtype=np.float64), inv_freq)
+
+
+def rope3d(x: np.ndarray, chunk: int, grid_h: int, grid_w: int,
+           frames_per_chunk: int, split, theta: float = 10000.0) -> np.ndarray:
+    """Return a rotated float64 copy of ``x`` ([tokens, heads, head_dim]).
+
+    head_dim is cut into segments [d_t | d_h | d_w] (``split``); in segment a
+    the pair (x[o+2j], x[o+2j+1]) turns by angle phi = pos_a * theta**(-2j/d_a):
+    (x0, x1) -> (x0 cos phi - x1 sin phi, x0 sin phi + x1 cos phi).
+    """
+    x = np.asarray(x, dtype=np.float64)
+    n_tok, _, dim = x.shape
+    d_t, d_h, d_w = (int(s) for s in split)
+    if d_t + d_h + d_w != dim or d_t % 2 or d_h % 2 or d_w % 2:
+        raise ValueError("rope split must be even and sum to head_dim")
+    f, r, col = token_positions(chunk, n_tok, grid_h, grid_w)
+    t = chunk * frames_per_chunk + f
+    out = x.copy()
+    offset = 0
+    for pos, width in ((t, d_t), (r, d_h), (col, d_w)):
+        if width:
+            ang = rope_angles(pos, width, theta)[:, None, :]  # [tok, 1, width/2]
+            c, s = np.cos(ang), np.sin(ang)
+            x0 = x[:, :, offset + 0: offset + width: 2]
+            x1 = x[:, :, offset + 1: offset + width: 2]
+            out[:, :, offset + 0: offset + width: 2] = x0 * c - x1 * s
+            out[:, :, offset + 1: offset + width: 2] = x0 * s + x1 * c
+        offset += width
+    return out
+
+
+# ---------------------------------------------------------------------------
+# Exact softmax attention (plain definition)
+# ---------------------------------------------------------------------------
+def attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float,
+              rows=None, return_probs: bool = False, row_block: int = 512):
+    """O[i,h,:] = sum_j softmax_j(scale * <q[i,h], k[j,h]>) v[j,h,:].
+
+    q: [Nq, H, D]; k, v: [Nkv, H, D] (float64). ``rows`` selects a subset of
+    query rows (sampled parity); ``None`` means all. Rows are independent, so
+    they are evaluated ``row_block`` at a time only to bound memory.
+    Returns out [len(rows), H, D] (and the probabilities [len(rows), H, Nkv]
+    when ``return_probs``).
+    """
+    q = np.asarray(q, dtype=np.float64)
+    k = np.asarray(k, dtype=np.float64)
+    v = np.asarray(v, dtype=np.float64)
+    rows = np.arange(q.shape[0]) if rows is None else np.asarray(rows, dtype=np.int64)
+    n_heads = q.shape[1]
+    out = np.empty((len(rows), n_heads, v.shape[2]), dtype=np.float64)
+    probs = np.empty((len(rows), n_heads, k.shape[0])) if return_probs else None
+    for h in range(n_heads):
+        kh = k[:, h, :]
+        vh = v[:, h, :]
+        for b0 in range(0, len(rows), row_block):
+            rb = rows[b0: b0 + row_block]
+            scores = scale * (q[rb, h, :] @ kh.T)          # [rows, Nkv]
+            m = scores.max(axis=1, keepdims=True)
+            e = np.exp(scores - m)
+            p = e / e.sum(axis=1, keepdims=True)
+            out[b0: b0 + len(rb), h, :] = p @ vh
+            if return_probs:
+                probs[b0: b0 + len(rb), h, :] = p
+    return (out, probs) if return_probs else out
+
+
+# ---------------------------------------------------------------------------
+# Sliding-window cache indices
+# ---------------------------------------------------------------------------
+def window_index(chunk: int, window: int):
+    """Ring slot written by ``chunk``, the chunk it evicts (-1 if none) and the
+    number of valid chunks after the append (window counts the current chunk)."""
+    if chunk < 0 or window < 1:
+        raise ValueError("chunk >= 0 and window >= 1 required")
+    slot = chunk % window
+    evicted = chunk - window if chunk >= window else -1
+    valid = min(chunk + 1, window)
+    return slot, evicted, valid
+
+
+class OracleStream:
+    """One stream's persistent state: a deque of the last W chunks of
+    (rotated K, V), i.e. the cross-batch KV-cache state edge of section 2.
+
+    ``step(q, k, v)`` runs one frame chunk: RoPE on q and k, append with
+    eviction, attention of the chunk's queries over the whole window.
+    """
+
+    def __init__(self, heads: int, head_dim: int, grid_h: int, grid_w: int,
+                 frames_per_chunk: int, window_chunks: int, split,
+                 theta: float = 10000.0, scale: float | None = None,
+                 exact: bool = False):
+        self.heads = heads
+        self.head_dim = head_dim
+        self.grid_h = grid_h
+        self.grid_w = grid_w
+        self.frames_per_chunk = frames_per_chunk
+        self.window = window_chunks
+        self.split = tuple(int(s) for s in split)
+        self.theta = float(theta)
+        self.scale = 1.0 / math.sqrt(head_dim) if scale is None else float(scale)
+        self.exact = exact
+        self.n_q = frames_per_chunk * grid_h * grid_w
+        self.chunk = 0
+        self.cache = collections.deque()  # entries: (chunk index, k_rot, v)
+
+    def rope(self, q, k):
+        """Rotate q and k at the current chunk's positions; round to bf16
+        unless ``exact``."""
+        args = (self.chunk, self.grid_h, self.grid_w, self.frames_per_chunk,
+                self.split, self.theta)
+        q_r = rope3d(q, *args)
+        k_r = rope3d(k, *args)
+        if not self.exact:
+            q_r, k_r = bf16_round(q_r), bf16_round(k_r)
+        return q_r, k_r
+
+    def append(self, k_rot, v):
+        """Append chunk ``self.chunk``; evict the chunk that leaves the window."""
+        slot, evicted, _ = window_index(self.chunk, self.window)
+        self.cache.append((self.chunk, np.asarray(k_rot, np.float64),
+                           np.asarray(v, np.float64)))
+        if len(self.cache) > self.window:
+            gone, _, _ = self.cache.popleft()
+            assert gone == evicted
+        self.chunk += 1
+        return slot, evicted
+
+    def cached_kv(self):
+        """Concatenation of every valid cached chunk's K and V, oldest first."""
+        k = np.concatenate([e[1] for e in self.cache], axis=0)
+        v = np.concatenate([e[2] for e in self.cache], axis=0)
+        return k, v
+
+    def attend(self, q_rot, rows=None, return_probs=False):
+        k, v = self.cached_kv()
+        return attention(q_rot, k, v, self.scale, rows=rows,
+                         return_probs=return_probs)
+
+    def step(self, q, k, v, rows=None):
+        """One frame chunk: (out, slot, evicted)."""
+        q_r, k_r = self.rope(q, k)
+        slot, evicted = self.append(k_r, v)
+        return self.attend(q_r, rows=rows), slot, evicted
