@@ -1,0 +1,453 @@
+"""Benchmark: streaming frame-chunk attention (3D RoPE + KV append/evict + chunk
+attention) on GB300, one JSON line on rank 0.
+
+A step is one frame chunk through the whole path (frt_chunk_step: RoPE-K fused into
+the append, RoPE-Q fused into the attention prologue) at steady state (full window).
+value = attention FLOPs of all ranks' steps / max-over-ranks wall time of the timed
+steps (CUDA events); ms_per_step = ms per frame chunk.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+                    [--impl reference]
+
+--impl reference times the fp64 CPU oracle on the host cores (a bounded row
+sample of the same workload per step). N > 1 runs under torchrun: one stream per
+rank, independent work (weak scaling), no data-path collective.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "chunk-attention TFLOP/s and ms per frame-chunk at 1 GB300; % of bf16 peak"
+UNIT = "TFLOP/s"
+POOL = 8  # distinct chunk inputs cycled through (larger than L2 for the 1.3B shape)
+
+
+def describe(wl) -> str:
+    return (f"{wl.name}: {wl.streams} stream(s), {wl.heads} heads x {wl.head_dim}, "
+            f"{wl.grid_h}x{wl.grid_w} latent grid, {wl.frames} frames/chunk (Nq {wl.n_q}), "
+            f"window {wl.window} chunks (Nkv {wl.window * wl.n_q} at steady state)")
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            pk = json.load(f)
+        return float(pk["bf16_tflops"]), float(pk["hbm_gbs"]), "measured"
+    except Exception:
+        return 1900.0, 6800.0, "fallback"
+
+
+def traffic_record(kernel_file: str, workload: str):
+    """DRAM bytes per launch from a committed ncu summary, only if the kernel source is
+    unchanged since the capture (sha256 of the .cu file recorded with the counters)."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    src = os.path.join(ROOT, "paper_2607_18171_gb300", "csrc", kernel_file)
+    try:
+        rec = json.load(open(path)).get(workload)
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()
+        if rec and rec.get("source_sha256") == sha:
+            return rec.get("dram_bytes_per_launch")
+    except Exception:
+        pass
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi samples during the timed region (clocks, throttle reasons)."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.proc = None
+        self.gpu = gpu_index
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-i", str(self.gpu), "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+                out = ""
+            self.lines = [l for l in out.splitlines() if l.strip()]
+        return False
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in getattr(self, "lines", []):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = float(parts[2])
+            except ValueError:
+                continue
+            for n, val in zip(names, parts[5:9]):
+                if val.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def init_dist():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def max_over_ranks(x: float, world: int, device) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------------------
+def run_gpu(args, wl, world, rank, local):
+    import torch
+    from paper_2607_18171_gb300 import frt, synth
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    frt.lib()
+    stream = torch.cuda.current_stream()
+    peak_tf, peak_gbs, peak_kind = load_peaks()
+
+    if wl.streams > 1:
+        return run_gpu_multi(args, wl, world, rank, local, dev, peak_tf, peak_kind)
+
+    sid = rank  # each rank streams its own independent video (weak scaling)
+    st = frt.Stream(wl.heads, wl.head_dim, wl.grid_h, wl.grid_w, wl.frames, wl.window,
+                    split=wl.split)
+    # prefill to a full window (untimed)
+    for c in range(wl.window - 1):
+        q, k, v = (t.to(dev) for t in synth.chunk_qkv(wl, sid, c))
+        st.chunk_step(q, k, v, st.new_out())
+    pool = [tuple(t.to(dev) for t in synth.chunk_qkv(wl, sid, wl.window - 1 + i))
+            for i in range(POOL)]
+    outs = [st.new_out() for _ in range(2)]
+    st.sync()
+    flops = wl.attn_flops(wl.window - 1)  # full window from here on
+
+    def step(i):
+        q, k, v = pool[i % POOL]
+        st.chunk_step(q, k, v, outs[i % 2])
+
+    for i in range(args.warmup):
+        step(i)
+    st.sync()
+    n = args.steps
+    ev_a = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+            for _ in range(n)]
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        t0.record(stream)
+        for i in range(n):
+            st.set_attention_events(*ev_a[i])
+            step(args.warmup + i)
+        t1.record(stream)
+        torch.cuda.synchronize()
+    st.set_attention_events(None, None)
+    st.sync()
+    if world > 1:
+        torch.distributed.barrier()
+    elapsed_ms = t0.elapsed_time(t1)
+    attn_ms = [a.elapsed_time(b) for a, b in ev_a]
+    wall_ms = max_over_ranks(elapsed_ms, world, dev)
+    total_flops = flops * n * world
+    value = total_flops / (wall_ms * 1e-3) / 1e12
+    attn_mean = statistics.mean(attn_ms)
+    achieved = flops / (attn_mean * 1e-3) / 1e12
+
+    # e2e through the host-buffer entry point: H2D of q,k,v + step + D2H of out
+    n_e2e = max(3, min(n, 50))
+    hq, hk, hv = (t.pin_memory() for t in synth.chunk_qkv(wl, sid, 1000))
+    hout = torch.empty(st.shape(), dtype=torch.float32).pin_memory()
+    for _ in range(2):
+        st.chunk_step_host(hq, hk, hv, hout)
+    st.sync()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(n_e2e):
+        st.chunk_step_host(hq, hk, hv, hout)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    e2e_value = flops * n_e2e * world / (e2e_ms * 1e-3) / 1e12
+    st.close()
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    if rank != 0:
+        return None
+
+    traffic = traffic_record("frt_attention.cu", wl.name)
+    line = {
+        "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
+        "steps": n, "warmup": args.warmup, "ms_per_step": round(wall_ms / n, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) bf16 Q/K/V shaped like the video-DiT workload)",
+        "config": {"workload": describe(wl), "path": "frt_chunk_step (RoPE-K in append, "
+                   "RoPE-Q in attention prologue)", "parallelism": f"independent streams x{world}",
+                   "l2": f"inputs larger than L2: {POOL} distinct chunk inputs "
+                   f"({POOL * 3 * wl.n_q * wl.heads * wl.head_dim * 2 / 1e6:.0f} MB) cycled, "
+                   f"KV cache {2 * wl.window * wl.n_q * wl.heads * wl.head_dim * 2 / 1e6:.0f} MB",
+                   "attn_flops_per_step": flops},
+        "roofline": {"bound": "tensor", "achieved": round(achieved, 2), "peak": peak_tf,
+                     "unit": "TFLOP/s", "frac": round(achieved / peak_tf, 4),
+                     "traffic": traffic, "kernel": "attn_kernel<128,1,true>",
+                     "peak_kind": f"{peak_kind} bf16 dense burst",
+                     "launch_ms": round(attn_mean, 4)},
+        "clocks": clk.summary(),
+        "e2e": {"value": round(e2e_value, 2), "unit": UNIT,
+                "h2d_bytes_per_step": 3 * wl.n_q * wl.heads * wl.head_dim * 2,
+                "d2h_bytes_per_step": wl.n_q * wl.heads * wl.head_dim * 4,
+                "steps": n_e2e, "ms_per_step": round(e2e_ms / n_e2e, 4)},
+        "gpu_launches": 2 * n,
+    }
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl, seconds=args.cpu_seconds)
+    return line
+
+
+def run_gpu_multi(args, wl, world, rank, local, dev, peak_tf, peak_kind):
+    """Ragged multi-stream step: per stream RoPE + append, then one batched attention
+    launch. Stream s keeps fill_s valid chunks (its window is fill_s), so the ragged KV
+    lengths persist across steps."""
+    import torch
+    from paper_2607_18171_gb300 import frt, synth
+
+    stream = torch.cuda.current_stream()
+    fills = synth.stream_fills(wl)
+    sts = []
+    for s, fill in enumerate(fills):
+        st = frt.Stream(wl.heads, wl.head_dim, wl.grid_h, wl.grid_w, wl.frames, fill,
+                        split=wl.split)
+        for c in range(fill - 1):
+            q, k, v = (t.to(dev) for t in synth.chunk_qkv(wl, 100 * rank + s, c))
+            st.chunk_step(q, k, v, st.new_out())
+        sts.append(st)
+    pool = [[tuple(t.to(dev) for t in synth.chunk_qkv(wl, 100 * rank + s, 50 + i))
+             for s in range(wl.streams)] for i in range(2)]
+    work = [[tuple(x.clone() for x in pool[i][s]) for s in range(wl.streams)] for i in range(2)]
+    outs = [st.new_out() for st in sts]
+    flops = sum(4 * wl.n_q * f * wl.n_q * wl.head_dim * wl.heads for f in fills)
+
+    def step(i):
+        w = work[i % 2]
+        for s, st in enumerate(sts):
+            q, k, v = w[s]
+            st.rope3d_qk(q, k)
+            st.kv_append_evict(k, v)
+        frt.chunk_attention_batched(sts, [w[s][0] for s in range(wl.streams)], outs)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    n = args.steps
+    ev_a = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+            for _ in range(n)]
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        t0.record(stream)
+        for i in range(n):
+            sts[0].set_attention_events(*ev_a[i])
+            step(args.warmup + i)
+        t1.record(stream)
+        torch.cuda.synchronize()
+    elapsed = max_over_ranks(t0.elapsed_time(t1), world, dev)
+    attn_mean = statistics.mean(a.elapsed_time(b) for a, b in ev_a)
+    for st in sts:
+        st.close()
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    if rank != 0:
+        return None
+    achieved = flops / (attn_mean * 1e-3) / 1e12
+    return {
+        "metric": METRIC, "value": round(flops * n * world / (elapsed * 1e-3) / 1e12, 2),
+        "unit": UNIT, "n_gpus": world, "steps": n, "warmup": args.warmup,
+        "ms_per_step": round(elapsed / n, 4), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": describe(wl) + f", fills {fills} (window = fill per stream)",
+                   "note": "step re-rotates the same two input sets in place; timing only"},
+        "roofline": {"bound": "tensor", "achieved": round(achieved, 2), "peak": peak_tf,
+                     "unit": "TFLOP/s", "frac": round(achieved / peak_tf, 4), "traffic": None,
+                     "kernel": "attn_kernel<128,32,false>", "peak_kind": peak_kind,
+                     "launch_ms": round(attn_mean, 4)},
+        "clocks": clk.summary(),
+        "gpu_launches": (2 * wl.streams + 1) * n,
+    }
+
+
+# ---------------------------------------------------------------------------------------
+# CPU oracle (baseline and reference arm)
+# ---------------------------------------------------------------------------------------
+def _oracle_stream(wl, sid, heads):
+    """Oracle state for the first ``heads`` heads of stream ``sid``, prefilled with the
+    window's first W-1 chunks (heads are independent, so a head subset is a faithful
+    sample of the computation)."""
+    from oracle.frt_oracle import OracleStream
+    from paper_2607_18171_gb300 import synth
+    orc = OracleStream(heads, wl.head_dim, wl.grid_h, wl.grid_w, wl.frames, wl.window,
+                       wl.split)
+    for c in range(wl.window - 1):
+        q, k, v = (synth.as_f64(t[:, :heads]) for t in synth.chunk_qkv(wl, sid, c))
+        q_r, k_r = orc.rope(q, k)
+        orc.append(k_r, v)
+    return orc
+
+
+def _oracle_step(orc, wl, sid, chunk, rows):
+    """Time one oracle chunk step (RoPE, append, attention of ``rows``)."""
+    from paper_2607_18171_gb300 import synth
+    h = orc.heads
+    q, k, v = (synth.as_f64(t[:, :h]) for t in synth.chunk_qkv(wl, sid, chunk))
+    t = time.perf_counter()
+    orc.step(q, k, v, rows=rows)
+    return time.perf_counter() - t
+
+
+def cpu_threads() -> int:
+    try:
+        import threadpoolctl
+        info = threadpoolctl.threadpool_info()
+        n = max((i.get("num_threads", 1) for i in info), default=0)
+        if n:
+            return int(n)
+    except Exception:
+        pass
+    return os.cpu_count() or 1
+
+
+def _rows_for(n_q, count):
+    return np.linspace(0, n_q - 1, max(1, min(n_q, int(count)))).astype(np.int64)
+
+
+def cpu_baseline(wl, seconds: float = 15.0):
+    """The oracle as it stands, on a bounded sample: one full-window chunk step (RoPE of
+    the chunk, append, exact fp64 attention) for all heads and a subset of query rows.
+    TFLOP/s = attention flops of the sampled rows / step time."""
+    if wl.streams > 1:
+        return None
+    orc = _oracle_stream(wl, 0, wl.heads)
+    nkv = wl.window * wl.n_q
+    probe = _rows_for(wl.n_q, 64)
+    dt = _oracle_step(orc, wl, 0, wl.window - 1, probe)      # window now full
+    rows = _rows_for(wl.n_q, len(probe) * seconds / max(dt, 1e-3))
+    dt = _oracle_step(orc, wl, 0, wl.window, rows)          # evicts chunk 0, still full
+    flops = 4 * len(rows) * nkv * wl.head_dim * wl.heads
+    return {"value": round(flops / dt / 1e12, 6), "unit": UNIT, "cores": cpu_threads(),
+            "kind": "oracle",
+            "sample": f"one full-window chunk step of {wl.name}: RoPE of the chunk + append + "
+                      f"exact fp64 attention for {len(rows)} of {wl.n_q} query rows x "
+                      f"{wl.heads} heads ({dt:.1f} s)"}
+
+
+def run_reference(args, wl, world, rank):
+    """Reference arm: the oracle timed as it stands on the host cores, one bounded
+    sample of the workload per step (one head, a row subset sized so the whole run
+    fits --ref-seconds)."""
+    if rank != 0:
+        return None
+    heads = 1
+    orc = _oracle_stream(wl, 0, heads)
+    nkv = wl.window * wl.n_q
+    probe = _rows_for(wl.n_q, 16)
+    dt = _oracle_step(orc, wl, 0, wl.window - 1, probe)
+    per_step = args.ref_seconds / max(1, args.steps + args.warmup)
+    rows = _rows_for(wl.n_q, len(probe) * per_step / max(dt, 1e-3))
+    times = []
+    for i in range(args.warmup + args.steps):
+        t = _oracle_step(orc, wl, 0, wl.window + i, rows)
+        if i >= args.warmup:
+            times.append(t)
+    total = sum(times)
+    flops = 4 * len(rows) * nkv * wl.head_dim * heads
+    value = flops * len(times) / total / 1e12
+    sample = (f"per step: one full-window chunk of {wl.name} (RoPE of the chunk, append, "
+              f"exact fp64 attention) for {len(rows)} of {wl.n_q} query rows x {heads} of "
+              f"{wl.heads} heads")
+    return {"metric": METRIC, "value": round(value, 6), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(1e3 * total / len(times), 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "impl": "reference", "config": {"workload": describe(wl)},
+            "cpu_baseline": {"value": round(value, 6), "unit": UNIT, "cores": cpu_threads(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(value, 6), "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--workload", default="dit1p3b")
+    ap.add_argument("--impl", default="frt", choices=["frt", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--ref-seconds", type=float, default=90.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    from paper_2607_18171_gb300 import synth
+    wl = synth.WORKLOADS[args.workload]
+    world, rank, local = init_dist()
+    if args.impl == "reference":
+        line = run_reference(args, wl, world, rank)
+    else:
+        line = run_gpu(args, wl, world, rank, local)
+    if line is not None:
+        print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

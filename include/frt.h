@@ -1,0 +1,182 @@
+/*
+ * frt.h — C ABI of the GB300 (sm_103a) streaming frame-chunk attention library.
+ *
+ * The workload is the per-chunk attention of an autoregressive video
+ * diffusion transformer over a persistent, rolling KV cache: the cache is the
+ * cross-batch state that batch j inherits from batch j-1 (arxiv 2607.18171,
+ * section 2 "Problem Formulation", the lambda = 1 state edge; Appendix A.1.2
+ * "Pipeline graph"), inputs arrive as frame chunks (Appendix A.1.1), and each
+ * denoising step owns an independent cache (section 3.1 "Case study";
+ * Appendix A.4), which here is one frt_stream_t per (request, step).
+ *
+ * One chunk c of a stream runs three operations, in this order:
+ *   1. 3D rotary embedding of q and k at the chunk's positions   (frt_rope3d_qk)
+ *   2. append of (k, v) to ring slot c mod W, evicting chunk c-W  (frt_kv_append_evict)
+ *   3. attention of the chunk's queries over every cached key     (frt_chunk_attention)
+ * or all three at once with frt_chunk_step (RoPE-Q runs inside the attention
+ * kernel's prologue, RoPE-K inside the append).
+ *
+ * Tensors: token-major [tokens, heads, head_dim], contiguous, bf16 for q/k/v,
+ * fp32 or bf16 for out, device pointers (unless a name ends in _host),
+ * 16-byte aligned. Token i of a chunk is frame i / (grid_h*grid_w), row
+ * (i mod grid_h*grid_w) / grid_w, column i mod grid_w.
+ *
+ * Ownership: the caller owns q/k/v/out; a stream owns its KV cache (allocated
+ * in frt_stream_configure, freed in frt_stream_destroy). A handle is not
+ * thread-safe; distinct handles are independent.
+ *
+ * Asynchrony: every call enqueues work on the stream's configured CUDA stream
+ * and returns after launch. Host-side argument and state errors are returned
+ * immediately and enqueue nothing. Device-side errors (a bounded wait that gave
+ * up) are recorded in a per-stream status word and returned by
+ * frt_stream_sync or by the next call on the stream.
+ */
+#ifndef FRT_H
+#define FRT_H
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct frt_stream frt_stream_t; /* opaque; owns its KV cache */
+
+typedef enum frt_status {
+    FRT_OK = 0,
+    FRT_ERR_INVALID_ARG = 1,  /* NULL/misaligned pointer, bad size or config */
+    FRT_ERR_STATE = 2,        /* call out of the rope -> append -> attention order */
+    FRT_ERR_OOM = 3,          /* device or pinned allocation failed */
+    FRT_ERR_CUDA = 4,         /* a CUDA runtime/driver call failed */
+    FRT_ERR_UNSUPPORTED = 5,  /* head_dim or shape the kernels do not handle */
+    FRT_ERR_TIMEOUT = 6       /* a device-side bounded wait gave up */
+} frt_status;
+
+typedef enum frt_out_dtype { FRT_OUT_F32 = 0, FRT_OUT_BF16 = 1 } frt_out_dtype;
+
+/* Per-stream configuration (frt_stream_configure). */
+typedef struct frt_config {
+    int grid_h, grid_w;            /* latent grid; grid_h * grid_w == tokens_per_frame */
+    int rope_dt, rope_dh, rope_dw; /* head_dim split [t | h | w]; each even, sum == head_dim */
+    double theta;                  /* RoPE base (10000) */
+    double sm_scale;               /* softmax scale; <= 0 selects 1/sqrt(head_dim) */
+    int out_dtype;                 /* frt_out_dtype */
+    void* cuda_stream;             /* cudaStream_t all work is enqueued on; NULL = legacy stream */
+} frt_config;
+
+/* Create a stream handle.
+ *   heads >= 1; head_dim in {64, 128}; tokens_per_frame >= 1;
+ *   frames_per_chunk >= 1; window_chunks >= 1 (the window counts the current chunk).
+ * Nq = frames_per_chunk * tokens_per_frame must be <= 2^20 and
+ * window_chunks * Nq <= 2^24. Allocates no device memory.
+ * Returns NULL on error; frt_last_error() then describes it. */
+frt_stream_t* frt_stream_create(int heads, int head_dim, int tokens_per_frame,
+                                int frames_per_chunk, int window_chunks);
+
+/* Fill *cfg with the defaults for s: grid 1 x tokens_per_frame, RoPE split
+ * (D/4, 3D/8, 3D/8) rounded to even, theta 10000, sm_scale 1/sqrt(D), fp32
+ * output, legacy CUDA stream. */
+frt_status frt_config_default(const frt_stream_t* s, frt_config* cfg);
+
+/* Validate and apply *cfg; allocates (once) and zero-fills the KV cache
+ * (2 * window_chunks * Nq * heads * head_dim bf16) and the RoPE tables, and
+ * resets the chunk counter to 0. Synchronous. Must precede every other call. */
+frt_status frt_stream_configure(frt_stream_t* s, const frt_config* cfg);
+
+/* Operation 1: rotate q and k (bf16 [Nq, heads, head_dim]) in place at the
+ * positions of chunk c = frt_stream_chunk_counter(s): token i sits at
+ * (t = c * frames_per_chunk + i / tokens_per_frame, row, column); in segment
+ * a of width d_a, pair (2j, 2j+1) turns by pos_a * theta^(-2j/d_a).
+ * Allowed at the start of a chunk (after configure/reset, an append, or an
+ * attention); otherwise FRT_ERR_STATE. */
+frt_status frt_rope3d_qk(frt_stream_t* s, void* q, void* k);
+
+/* Operation 2: copy the rotated k and v of chunk c into ring slot c mod W
+ * (cache rows [slot*Nq, (slot+1)*Nq)), overwriting evicted chunk c - W, then
+ * advance the counter. *slot_out = c mod W, *evicted_out = c - W or -1 (either
+ * pointer may be NULL). Indices are computed on the host (exact). Must follow
+ * frt_rope3d_qk of the same chunk; otherwise FRT_ERR_STATE. */
+frt_status frt_kv_append_evict(frt_stream_t* s, const void* k, const void* v,
+                               int* slot_out, long long* evicted_out);
+
+/* Operation 3: out[i, h, :] = sum_j softmax_j(sm_scale * <q[i,h], K[j,h]>) V[j,h,:]
+ * over every valid cached row j (n_c * Nq rows, n_c = min(c + 1, W) for the
+ * chunk c just appended): bidirectional inside the chunk, all earlier chunks
+ * of the window. bf16 operands, fp32 accumulation, P rounded to bf16 for the
+ * PV product. q must be the pointer rotated by the last frt_rope3d_qk; k and v
+ * must be the pointers of the last append, or NULL (K/V are read from the
+ * cache either way). out: [Nq, heads, head_dim] in the configured dtype.
+ * Must follow an append; otherwise FRT_ERR_STATE. */
+frt_status frt_chunk_attention(const void* q, const void* k, const void* v,
+                               void* out, frt_stream_t* s);
+
+/* Operations 1-3 fused for one chunk: q, k, v are the raw (unrotated) inputs
+ * and are not modified; RoPE-K runs inside the append (rotated K goes to the
+ * cache only) and RoPE-Q inside the attention kernel's prologue. Same result
+ * as the three separate calls. Allowed at the start of a chunk. */
+frt_status frt_chunk_step(frt_stream_t* s, const void* q, const void* k,
+                          const void* v, void* out, int* slot_out,
+                          long long* evicted_out);
+
+/* frt_chunk_step with HOST buffers: copies q, k, v host -> device into
+ * stream-owned staging buffers, runs the fused step, copies out device ->
+ * host, all enqueued on the stream. Host buffers must stay valid until
+ * frt_stream_sync returns (pinned memory makes the copies asynchronous). */
+frt_status frt_chunk_step_host(frt_stream_t* s, const void* q_host,
+                               const void* k_host, const void* v_host,
+                               void* out_host, int* slot_out,
+                               long long* evicted_out);
+
+/* Operation 3 for n independent streams in one launch (ragged KV lengths):
+ * each streams[i] must have just appended (as for frt_chunk_attention); q[i]
+ * and out[i] are that stream's rotated queries and output. All streams must
+ * share heads, head_dim, sm_scale and out dtype; work is ordered longest KV
+ * first and enqueued on streams[0]'s CUDA stream, which first waits for the
+ * other streams' CUDA streams (events), and which they wait for afterwards.
+ * 1 <= n <= 32, no stream repeated. */
+frt_status frt_chunk_attention_batched(frt_stream_t* const* streams, int n,
+                                       const void* const* q, void* const* out);
+
+/* Wait for the stream's work and return its device status (FRT_OK or the
+ * first device error, e.g. FRT_ERR_TIMEOUT). */
+frt_status frt_stream_sync(frt_stream_t* s);
+
+/* Clear the cache contents, chunk counter, ordering state and device status. */
+frt_status frt_stream_reset(frt_stream_t* s);
+
+/* Release everything the handle owns (waits for its work first). NULL is a no-op. */
+void frt_stream_destroy(frt_stream_t* s);
+
+/* Read-only view of the stream's ring buffer for inspection and snapshots: device
+ * pointers of the K and V caches ([rows, heads, head_dim] bf16, rows = W * Nq; chunk c
+ * occupies rows [(c mod W) * Nq, (c mod W + 1) * Nq)). Valid until destroy. */
+frt_status frt_stream_cache(const frt_stream_t* s, const void** k_cache,
+                            const void** v_cache, long long* rows);
+
+/* Instrumentation: record start_event / stop_event (cudaEvent_t, created by the
+ * caller) on the stream's CUDA stream immediately before and after every
+ * attention kernel launch of s (frt_chunk_attention, frt_chunk_step and batched
+ * launches led by s) until called again; NULL, NULL turns it off. */
+frt_status frt_stream_set_attention_events(frt_stream_t* s, void* start_event,
+                                           void* stop_event);
+
+/* Index of the next chunk to be appended (chunks appended so far). */
+long long frt_stream_chunk_counter(const frt_stream_t* s);
+
+/* Host-only sliding-window arithmetic used by frt_kv_append_evict: for chunk
+ * index `chunk` >= 0 and window >= 1, the ring slot (chunk mod window), the
+ * evicted chunk (chunk - window, or -1) and the valid chunk count after the
+ * append (min(chunk + 1, window)). Any output pointer may be NULL. */
+frt_status frt_window_index(long long chunk, int window, int* slot,
+                            long long* evicted, int* valid_chunks);
+
+const char* frt_status_string(frt_status st);
+
+/* Thread-local description of the last error returned on this thread. */
+const char* frt_last_error(void);
+
+/* Library version string. */
+const char* frt_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* FRT_H */

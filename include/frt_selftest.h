@@ -1,0 +1,33 @@
+/*
+ * frt_selftest.h — self-test entry points of libfrt.so, used by the GPU tests to
+ * check the hardware building blocks of the attention kernel in isolation. They are
+ * not part of the streaming API (include/frt.h) and have no counterpart in the paper.
+ */
+#ifndef FRT_SELFTEST_H
+#define FRT_SELFTEST_H
+#include "frt.h"
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* One 128x128x128 bf16 tile, C = A * op(B), fp32, through TMA (128-byte swizzle) into
+ * shared memory, tcgen05.mma into TMEM and tcgen05.ld back to registers.
+ *   a: device [128, 128] bf16 row-major (row m, reduction index k contiguous).
+ *   b: device [128, 128] bf16 row-major; b_mn_major = 0: b[n][k] (C = A B^T, the QK^T
+ *      layout); b_mn_major = 1: b[k][n] (C = A B, the PV layout).
+ *   lbo_b, sbo_b: descriptor byte offsets for the MN-major B (16 <= x <= 16384).
+ *   a_from_tmem: 1 stages A in TMEM (packed bf16 pairs) and uses the A-from-TMEM MMA.
+ *   c: device [128, 128] fp32 row-major; dev_status: device int set to 1 on a timeout.
+ * Enqueued on cuda_stream; returns 0 on launch success, < 0 on an argument/launch error. */
+int frt_selftest_umma_tile(const void* a, const void* b, float* c, int b_mn_major, int lbo_b,
+                           int sbo_b, int a_from_tmem, int* dev_status, void* cuda_stream);
+
+/* Launch a kernel whose one waiting thread waits on an mbarrier that nothing arrives
+ * on, bounded by limit_ns (<= 100 ms); it must record FRT_ERR_TIMEOUT in s's status
+ * block, which frt_stream_sync then returns. s must be configured. */
+frt_status frt_selftest_wait_timeout(frt_stream_t* s, long long limit_ns, void* cuda_stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

@@ -149,19 +149,18 @@ def attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float,
     Returns out [len(rows), H, D] (and the probabilities [len(rows), H, Nkv]
     when ``return_probs``).
     """
-    q = np.asarray(q, dtype=np.float64)
-    k = np.asarray(k, dtype=np.float64)
-    v = np.asarray(v, dtype=np.float64)
     rows = np.arange(q.shape[0]) if rows is None else np.asarray(rows, dtype=np.int64)
     n_heads = q.shape[1]
     out = np.empty((len(rows), n_heads, v.shape[2]), dtype=np.float64)
     probs = np.empty((len(rows), n_heads, k.shape[0])) if return_probs else None
     for h in range(n_heads):
-        kh = k[:, h, :]
-        vh = v[:, h, :]
+        # widen one head at a time (inputs may be float32 holding bf16 values exactly)
+        kh = np.asarray(k[:, h, :], dtype=np.float64)
+        vh = np.asarray(v[:, h, :], dtype=np.float64)
         for b0 in range(0, len(rows), row_block):
             rb = rows[b0: b0 + row_block]
-            scores = scale * (q[rb, h, :] @ kh.T)          # [rows, Nkv]
+            qh = np.asarray(q[rb, h, :], dtype=np.float64)
+            scores = scale * (qh @ kh.T)                    # [rows, Nkv]
             m = scores.max(axis=1, keepdims=True)
             e = np.exp(scores - m)
             p = e / e.sum(axis=1, keepdims=True)

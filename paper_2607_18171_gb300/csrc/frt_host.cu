@@ -1,0 +1,616 @@
+// frt_host.cu — the C ABI (include/frt.h): per-stream persistent state (the rolling KV
+// cache), host-side window arithmetic, argument/state checks, TMA descriptor encoding and
+// kernel launches on the caller's CUDA stream.
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "../../include/frt.h"
+#include "frt_internal.h"
+
+using namespace frt;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+frt_status fail(frt_status st, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return st;
+}
+
+frt_status cuda_fail(cudaError_t e, const char* what) {
+    return fail(e == cudaErrorMemoryAllocation ? FRT_ERR_OOM : FRT_ERR_CUDA, "%s: %s", what,
+                cudaGetErrorString(e));
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+// 3D map over a token-major [rows, heads, head_dim] bf16 tensor; box = 64 dims x 1 head x
+// 128 rows, 128-byte swizzle; rows past `rows` read as zero.
+frt_status make_map(CUtensorMap* map, const void* base, int head_dim, int heads, long long rows) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return fail(FRT_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+    cuuint64_t dims[3] = {cuuint64_t(head_dim), cuuint64_t(heads), cuuint64_t(rows)};
+    cuuint64_t strides[2] = {cuuint64_t(head_dim) * 2, cuuint64_t(heads) * head_dim * 2};
+    cuuint32_t box[3] = {64, 1, 128};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims,
+                    strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(FRT_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", int(r));
+    return FRT_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+enum Phase { kStart = 0, kRoped = 1, kAppended = 2 };
+
+constexpr unsigned long long kDefaultWaitLimitNs = 2000000000ull;  // 2 s per bounded wait
+
+}  // namespace
+
+struct frt_stream {
+    int heads, head_dim, tpf, frames, window, n_q;
+    bool configured = false;
+    frt_config cfg{};
+    float scale = 0.f;
+    cudaStream_t cs = nullptr;
+    void* cache_k = nullptr;
+    void* cache_v = nullptr;
+    size_t chunk_elems = 0;     // Nq * H * D
+    float2* d_hw = nullptr;     // h/w RoPE tables
+    int hw_entries = 0;
+    DeviceStatus* status_host = nullptr;
+    DeviceStatus* status_dev = nullptr;
+    long long counter = 0;
+    int phase = kStart;
+    const void* last_q = nullptr;
+    const void* last_k = nullptr;
+    const void* last_v = nullptr;
+    void* stage = nullptr;      // host-API staging: q, k, v (bf16) and out
+    size_t stage_bytes = 0;
+    unsigned long long wait_limit_ns = kDefaultWaitLimitNs;
+    cudaEvent_t ev = nullptr;   // cross-stream ordering for batched launches
+    cudaEvent_t attn_start = nullptr;  // caller-owned instrumentation events
+    cudaEvent_t attn_stop = nullptr;
+};
+
+namespace {
+
+frt_status check_device_status(frt_stream_t* s) {
+    if (s->status_host == nullptr) return FRT_OK;
+    volatile DeviceStatus* st = s->status_host;
+    int code = st->code;
+    if (code != 0)
+        return fail(static_cast<frt_status>(code),
+                    "device wait gave up (block %d, role %d, at %d); reset the stream", st->block,
+                    st->role, st->where);
+    return FRT_OK;
+}
+
+frt_status require_configured(frt_stream_t* s) {
+    if (s == nullptr) return fail(FRT_ERR_INVALID_ARG, "NULL stream handle");
+    if (!s->configured) return fail(FRT_ERR_STATE, "stream not configured");
+    return check_device_status(s);
+}
+
+// RoPE argument block for chunk `c` (t-segment cos/sin of its frames, fp64 -> fp32).
+void fill_rope(const frt_stream_t* s, long long c, RopeArgs& a) {
+    a.hw = s->d_hw;
+    a.tpf = s->tpf;
+    a.gh = s->cfg.grid_h;
+    a.gw = s->cfg.grid_w;
+    a.dt2 = s->cfg.rope_dt / 2;
+    a.dh2 = s->cfg.rope_dh / 2;
+    a.dw2 = s->cfg.rope_dw / 2;
+    const double theta = s->cfg.theta;
+    for (int f = 0; f < s->frames; ++f) {
+        const double t = double(c) * s->frames + f;
+        for (int j = 0; j < a.dt2; ++j) {
+            const double ang = t * std::pow(theta, -2.0 * j / double(s->cfg.rope_dt));
+            a.t_tab[f * a.dt2 + j] = make_float2(float(std::cos(ang)), float(std::sin(ang)));
+        }
+    }
+}
+
+int log2_exact(int x) {
+    int l = 0;
+    while ((1 << l) < x) ++l;
+    return l;
+}
+
+frt_status attention_single(frt_stream_t* s, const void* q, void* out, bool rope_q) {
+    AttnParams<1> p;
+    std::memset(&p, 0, sizeof(p));
+    const long long n_valid = std::min<long long>(s->counter, s->window);
+    AttnStreamDesc& d = p.s[0];
+    frt_status st;
+    if ((st = make_map(&d.q_map, q, s->head_dim, s->heads, s->n_q)) != FRT_OK) return st;
+    const long long n_kv = n_valid * s->n_q;
+    if ((st = make_map(&d.k_map, s->cache_k, s->head_dim, s->heads, n_kv)) != FRT_OK) return st;
+    if ((st = make_map(&d.v_map, s->cache_v, s->head_dim, s->heads, n_kv)) != FRT_OK) return st;
+    d.out = out;
+    d.n_q = s->n_q;
+    d.n_kv = int(n_kv);
+    d.n_qpairs = (s->n_q + 255) / 256;
+    d.item_begin = 0;
+    p.n_streams = 1;
+    p.heads = s->heads;
+    p.total_items = d.n_qpairs * s->heads;
+    p.out_bf16 = s->cfg.out_dtype == FRT_OUT_BF16;
+    p.scale_log2 = float(double(s->scale) * 1.4426950408889634);
+    p.wait_limit_ns = s->wait_limit_ns;
+    p.status = s->status_dev;
+    if (rope_q) fill_rope(s, s->counter - 1, p.rope);
+    cudaError_t e = cudaSuccess;
+    if (s->attn_start) e = cudaEventRecord(s->attn_start, s->cs);
+    if (e == cudaSuccess) e = launch_attention_single(p, s->head_dim, rope_q, s->cs);
+    if (e == cudaSuccess && s->attn_stop) e = cudaEventRecord(s->attn_stop, s->cs);
+    if (e != cudaSuccess) return cuda_fail(e, "attention launch");
+    return FRT_OK;
+}
+
+frt_status append_impl(frt_stream_t* s, const void* k, const void* v, bool rope_k, int* slot_out,
+                       long long* evicted_out) {
+    int slot;
+    long long evicted;
+    frt_window_index(s->counter, s->window, &slot, &evicted, nullptr);
+    AppendParams p;
+    std::memset(&p, 0, sizeof(p));
+    const size_t off = size_t(slot) * s->chunk_elems;
+    p.k_src = static_cast<const uint4*>(k);
+    p.v_src = static_cast<const uint4*>(v);
+    p.k_dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(s->cache_k) + off);
+    p.v_dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(s->cache_v) + off);
+    p.n_tok = s->n_q;
+    p.vec_per_tok = s->heads * s->head_dim / 8;
+    p.vec_per_head_log2 = log2_exact(s->head_dim / 8);
+    p.rope = rope_k ? 1 : 0;
+    if (rope_k) fill_rope(s, s->counter, p.ra);
+    cudaError_t e = launch_kv_append(p, s->cs);
+    if (e != cudaSuccess) return cuda_fail(e, "append launch");
+    s->counter += 1;
+    s->phase = kAppended;
+    s->last_k = k;
+    s->last_v = v;
+    if (slot_out) *slot_out = slot;
+    if (evicted_out) *evicted_out = evicted;
+    return FRT_OK;
+}
+
+void free_device(frt_stream_t* s) {
+    if (s->cache_k) cudaFree(s->cache_k);
+    if (s->cache_v) cudaFree(s->cache_v);
+    if (s->d_hw) cudaFree(s->d_hw);
+    if (s->stage) cudaFree(s->stage);
+    if (s->status_host) cudaFreeHost(s->status_host);
+    if (s->ev) cudaEventDestroy(s->ev);
+    s->ev = nullptr;
+    s->cache_k = s->cache_v = nullptr;
+    s->d_hw = nullptr;
+    s->stage = nullptr;
+    s->status_host = s->status_dev = nullptr;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* frt_version(void) { return "frt 0.1 (sm_103a)"; }
+
+const char* frt_last_error(void) { return g_last_error.c_str(); }
+
+const char* frt_status_string(frt_status st) {
+    switch (st) {
+        case FRT_OK: return "FRT_OK";
+        case FRT_ERR_INVALID_ARG: return "FRT_ERR_INVALID_ARG";
+        case FRT_ERR_STATE: return "FRT_ERR_STATE";
+        case FRT_ERR_OOM: return "FRT_ERR_OOM";
+        case FRT_ERR_CUDA: return "FRT_ERR_CUDA";
+        case FRT_ERR_UNSUPPORTED: return "FRT_ERR_UNSUPPORTED";
+        case FRT_ERR_TIMEOUT: return "FRT_ERR_TIMEOUT";
+    }
+    return "FRT_ERR_UNKNOWN";
+}
+
+frt_status frt_window_index(long long chunk, int window, int* slot, long long* evicted,
+                            int* valid_chunks) {
+    if (chunk < 0 || window < 1) return fail(FRT_ERR_INVALID_ARG, "chunk >= 0 and window >= 1");
+    if (slot) *slot = int(chunk % window);
+    if (evicted) *evicted = chunk >= window ? chunk - window : -1;
+    if (valid_chunks) *valid_chunks = int(chunk + 1 < window ? chunk + 1 : window);
+    return FRT_OK;
+}
+
+frt_stream_t* frt_stream_create(int heads, int head_dim, int tokens_per_frame,
+                                int frames_per_chunk, int window_chunks) {
+    if (heads < 1 || tokens_per_frame < 1 || frames_per_chunk < 1 || window_chunks < 1) {
+        fail(FRT_ERR_INVALID_ARG, "heads, tokens_per_frame, frames_per_chunk, window >= 1");
+        return nullptr;
+    }
+    if (head_dim != 64 && head_dim != 128) {
+        fail(FRT_ERR_UNSUPPORTED, "head_dim %d unsupported (64 or 128)", head_dim);
+        return nullptr;
+    }
+    const long long n_q = (long long)frames_per_chunk * tokens_per_frame;
+    if (n_q > (1 << 20) || n_q * window_chunks > (1 << 24) || heads > 1024) {
+        fail(FRT_ERR_UNSUPPORTED, "chunk or window too large (Nq=%lld, W=%d)", n_q, window_chunks);
+        return nullptr;
+    }
+    frt_stream_t* s = new (std::nothrow) frt_stream();
+    if (!s) {
+        fail(FRT_ERR_OOM, "host allocation failed");
+        return nullptr;
+    }
+    s->heads = heads;
+    s->head_dim = head_dim;
+    s->tpf = tokens_per_frame;
+    s->frames = frames_per_chunk;
+    s->window = window_chunks;
+    s->n_q = int(n_q);
+    s->chunk_elems = size_t(n_q) * heads * head_dim;
+    frt_config_default(s, &s->cfg);
+    return s;
+}
+
+frt_status frt_config_default(const frt_stream_t* s, frt_config* cfg) {
+    if (!s || !cfg) return fail(FRT_ERR_INVALID_ARG, "NULL argument");
+    const int D = s->head_dim;
+    int dt = 2 * int(std::lround(D / 8.0));
+    int dh = 2 * ((D - dt) / 4);
+    cfg->grid_h = 1;
+    cfg->grid_w = s->tpf;
+    cfg->rope_dt = dt;
+    cfg->rope_dh = dh;
+    cfg->rope_dw = D - dt - dh;
+    cfg->theta = 10000.0;
+    cfg->sm_scale = 1.0 / std::sqrt(double(D));
+    cfg->out_dtype = FRT_OUT_F32;
+    cfg->cuda_stream = nullptr;
+    return FRT_OK;
+}
+
+frt_status frt_stream_configure(frt_stream_t* s, const frt_config* cfg) {
+    if (!s || !cfg) return fail(FRT_ERR_INVALID_ARG, "NULL argument");
+    if (cfg->grid_h < 1 || cfg->grid_w < 1 || (long long)cfg->grid_h * cfg->grid_w != s->tpf)
+        return fail(FRT_ERR_INVALID_ARG, "grid_h * grid_w must equal tokens_per_frame");
+    if (cfg->rope_dt < 0 || cfg->rope_dh < 0 || cfg->rope_dw < 0 || (cfg->rope_dt & 1) ||
+        (cfg->rope_dh & 1) || (cfg->rope_dw & 1) ||
+        cfg->rope_dt + cfg->rope_dh + cfg->rope_dw != s->head_dim)
+        return fail(FRT_ERR_INVALID_ARG, "rope split must be even and sum to head_dim");
+    if (!(cfg->theta > 1.0)) return fail(FRT_ERR_INVALID_ARG, "theta must be > 1");
+    if (cfg->out_dtype != FRT_OUT_F32 && cfg->out_dtype != FRT_OUT_BF16)
+        return fail(FRT_ERR_INVALID_ARG, "unknown out_dtype");
+    if ((long long)s->frames * (cfg->rope_dt / 2) > kMaxTEntries)
+        return fail(FRT_ERR_UNSUPPORTED, "frames_per_chunk * d_t/2 exceeds %d", kMaxTEntries);
+    if (s->configured) {
+        cudaError_t e = cudaStreamSynchronize(s->cs);
+        if (e != cudaSuccess) return cuda_fail(e, "sync before reconfigure");
+    }
+    s->cfg = *cfg;
+    s->scale = float(cfg->sm_scale > 0 ? cfg->sm_scale : 1.0 / std::sqrt(double(s->head_dim)));
+    s->cs = static_cast<cudaStream_t>(cfg->cuda_stream);
+
+    cudaError_t e;
+    const size_t cache_bytes = size_t(s->window) * s->chunk_elems * 2;
+    if (!s->cache_k) {
+        if ((e = cudaMalloc(&s->cache_k, cache_bytes)) != cudaSuccess ||
+            (e = cudaMalloc(&s->cache_v, cache_bytes)) != cudaSuccess) {
+            free_device(s);
+            return cuda_fail(e, "cache allocation");
+        }
+    }
+    if (!s->status_host) {
+        if ((e = cudaHostAlloc(reinterpret_cast<void**>(&s->status_host), sizeof(DeviceStatus),
+                               cudaHostAllocMapped)) != cudaSuccess ||
+            (e = cudaHostGetDevicePointer(reinterpret_cast<void**>(&s->status_dev),
+                                          s->status_host, 0)) != cudaSuccess) {
+            free_device(s);
+            return cuda_fail(e, "status allocation");
+        }
+    }
+    std::memset(s->status_host, 0, sizeof(DeviceStatus));
+    if (!s->ev && (e = cudaEventCreateWithFlags(&s->ev, cudaEventDisableTiming)) != cudaSuccess) {
+        free_device(s);
+        return cuda_fail(e, "event creation");
+    }
+    // h/w tables: [grid_h][d_h/2] then [grid_w][d_w/2], cos/sin computed in fp64
+    const int dh2 = cfg->rope_dh / 2, dw2 = cfg->rope_dw / 2;
+    std::vector<float2> hw(size_t(cfg->grid_h) * dh2 + size_t(cfg->grid_w) * dw2 + 1);
+    for (int r = 0; r < cfg->grid_h; ++r)
+        for (int j = 0; j < dh2; ++j) {
+            const double a = r * std::pow(cfg->theta, -2.0 * j / double(cfg->rope_dh));
+            hw[size_t(r) * dh2 + j] = make_float2(float(std::cos(a)), float(std::sin(a)));
+        }
+    for (int c = 0; c < cfg->grid_w; ++c)
+        for (int j = 0; j < dw2; ++j) {
+            const double a = c * std::pow(cfg->theta, -2.0 * j / double(cfg->rope_dw));
+            hw[size_t(cfg->grid_h) * dh2 + size_t(c) * dw2 + j] =
+                make_float2(float(std::cos(a)), float(std::sin(a)));
+        }
+    if (s->d_hw) cudaFree(s->d_hw);
+    s->d_hw = nullptr;
+    if ((e = cudaMalloc(&s->d_hw, hw.size() * sizeof(float2))) != cudaSuccess) {
+        free_device(s);
+        return cuda_fail(e, "rope table allocation");
+    }
+    if ((e = cudaMemcpy(s->d_hw, hw.data(), hw.size() * sizeof(float2),
+                        cudaMemcpyHostToDevice)) != cudaSuccess)
+        return cuda_fail(e, "rope table upload");
+    s->hw_entries = int(hw.size());
+    // zero cache: rows past the valid prefix are never read by value, but keep them finite
+    if ((e = cudaMemset(s->cache_k, 0, cache_bytes)) != cudaSuccess ||
+        (e = cudaMemset(s->cache_v, 0, cache_bytes)) != cudaSuccess)
+        return cuda_fail(e, "cache clear");
+    if ((e = cudaDeviceSynchronize()) != cudaSuccess) return cuda_fail(e, "configure sync");
+    s->counter = 0;
+    s->phase = kStart;
+    s->last_q = s->last_k = s->last_v = nullptr;
+    s->configured = true;
+    return FRT_OK;
+}
+
+frt_status frt_rope3d_qk(frt_stream_t* s, void* q, void* k) {
+    frt_status st = require_configured(s);
+    if (st != FRT_OK) return st;
+    if (!q || !k || !aligned16(q) || !aligned16(k))
+        return fail(FRT_ERR_INVALID_ARG, "q and k must be non-NULL and 16-byte aligned");
+    if (s->phase == kRoped) return fail(FRT_ERR_STATE, "rope called twice for one chunk");
+    RopeParams p;
+    std::memset(&p, 0, sizeof(p));
+    p.q = static_cast<uint4*>(q);
+    p.k = static_cast<uint4*>(k);
+    p.n_tok = s->n_q;
+    p.vec_per_tok = s->heads * s->head_dim / 8;
+    p.vec_per_head_log2 = log2_exact(s->head_dim / 8);
+    fill_rope(s, s->counter, p.ra);
+    cudaError_t e = launch_rope_qk(p, s->cs);
+    if (e != cudaSuccess) return cuda_fail(e, "rope launch");
+    s->phase = kRoped;
+    s->last_q = q;
+    return FRT_OK;
+}
+
+frt_status frt_kv_append_evict(frt_stream_t* s, const void* k, const void* v, int* slot_out,
+                               long long* evicted_out) {
+    frt_status st = require_configured(s);
+    if (st != FRT_OK) return st;
+    if (!k || !v || !aligned16(k) || !aligned16(v))
+        return fail(FRT_ERR_INVALID_ARG, "k and v must be non-NULL and 16-byte aligned");
+    if (s->phase != kRoped) return fail(FRT_ERR_STATE, "append must follow frt_rope3d_qk");
+    return append_impl(s, k, v, false, slot_out, evicted_out);
+}
+
+frt_status frt_chunk_attention(const void* q, const void* k, const void* v, void* out,
+                               frt_stream_t* s) {
+    frt_status st = require_configured(s);
+    if (st != FRT_OK) return st;
+    if (!q || !out || !aligned16(q) || !aligned16(out))
+        return fail(FRT_ERR_INVALID_ARG, "q and out must be non-NULL and 16-byte aligned");
+    if (s->phase != kAppended) return fail(FRT_ERR_STATE, "attention must follow an append");
+    if ((k && k != s->last_k) || (v && v != s->last_v))
+        return fail(FRT_ERR_STATE, "k/v are not the tensors of the last append");
+    if (q != s->last_q) return fail(FRT_ERR_STATE, "q is not the tensor rotated for this chunk");
+    return attention_single(s, q, out, false);
+}
+
+frt_status frt_chunk_step(frt_stream_t* s, const void* q, const void* k, const void* v,
+                          void* out, int* slot_out, long long* evicted_out) {
+    frt_status st = require_configured(s);
+    if (st != FRT_OK) return st;
+    if (!q || !k || !v || !out || !aligned16(q) || !aligned16(k) || !aligned16(v) ||
+        !aligned16(out))
+        return fail(FRT_ERR_INVALID_ARG, "q, k, v, out must be non-NULL and 16-byte aligned");
+    if (s->phase == kRoped) return fail(FRT_ERR_STATE, "a separate rope is pending");
+    if ((st = append_impl(s, k, v, true, slot_out, evicted_out)) != FRT_OK) return st;
+    s->last_q = q;
+    return attention_single(s, q, out, true);
+}
+
+frt_status frt_chunk_step_host(frt_stream_t* s, const void* q_host, const void* k_host,
+                               const void* v_host, void* out_host, int* slot_out,
+                               long long* evicted_out) {
+    frt_status st = require_configured(s);
+    if (st != FRT_OK) return st;
+    if (!q_host || !k_host || !v_host || !out_host)
+        return fail(FRT_ERR_INVALID_ARG, "NULL host buffer");
+    const size_t in_bytes = s->chunk_elems * 2;
+    const size_t out_bytes = s->chunk_elems * (s->cfg.out_dtype == FRT_OUT_BF16 ? 2 : 4);
+    const size_t need = 3 * in_bytes + out_bytes;
+    cudaError_t e;
+    if (s->stage_bytes < need) {
+        if (s->stage) {
+            if ((e = cudaStreamSynchronize(s->cs)) != cudaSuccess) return cuda_fail(e, "sync");
+            cudaFree(s->stage);
+            s->stage = nullptr;
+            s->stage_bytes = 0;
+        }
+        if ((e = cudaMalloc(&s->stage, need)) != cudaSuccess) return cuda_fail(e, "staging");
+        s->stage_bytes = need;
+    }
+    uint8_t* base = static_cast<uint8_t*>(s->stage);
+    void* dq = base;
+    void* dk = base + in_bytes;
+    void* dv = base + 2 * in_bytes;
+    void* dout = base + 3 * in_bytes;
+    if ((e = cudaMemcpyAsync(dq, q_host, in_bytes, cudaMemcpyHostToDevice, s->cs)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(dk, k_host, in_bytes, cudaMemcpyHostToDevice, s->cs)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(dv, v_host, in_bytes, cudaMemcpyHostToDevice, s->cs)) != cudaSuccess)
+        return cuda_fail(e, "host-to-device copy");
+    if ((st = frt_chunk_step(s, dq, dk, dv, dout, slot_out, evicted_out)) != FRT_OK) return st;
+    if ((e = cudaMemcpyAsync(out_host, dout, out_bytes, cudaMemcpyDeviceToHost, s->cs)) !=
+        cudaSuccess)
+        return cuda_fail(e, "device-to-host copy");
+    return FRT_OK;
+}
+
+frt_status frt_chunk_attention_batched(frt_stream_t* const* streams, int n, const void* const* q,
+                                       void* const* out) {
+    if (!streams || !q || !out || n < 1 || n > kMaxBatchStreams)
+        return fail(FRT_ERR_INVALID_ARG, "need 1 <= n <= %d streams and q/out arrays",
+                    kMaxBatchStreams);
+    frt_stream_t* s0 = streams[0];
+    frt_status st;
+    for (int i = 0; i < n; ++i) {
+        frt_stream_t* s = streams[i];
+        if ((st = require_configured(s)) != FRT_OK) return st;
+        if (s->heads != s0->heads || s->head_dim != s0->head_dim || s->scale != s0->scale ||
+            s->cfg.out_dtype != s0->cfg.out_dtype)
+            return fail(FRT_ERR_UNSUPPORTED, "batched streams must share heads, head_dim, scale, dtype");
+        if (s->phase != kAppended) return fail(FRT_ERR_STATE, "stream %d has not appended", i);
+        if (!q[i] || !out[i] || !aligned16(q[i]) || !aligned16(out[i]))
+            return fail(FRT_ERR_INVALID_ARG, "q/out %d NULL or misaligned", i);
+        if (q[i] != s->last_q) return fail(FRT_ERR_STATE, "q %d is not this chunk's rotated q", i);
+        for (int j = 0; j < i; ++j)
+            if (streams[j] == s) return fail(FRT_ERR_INVALID_ARG, "stream %d repeated", i);
+    }
+    // longest KV first (LPT): items are handed to SMs in launch order
+    std::vector<int> order(n);
+    for (int i = 0; i < n; ++i) order[i] = i;
+    auto n_kv = [&](int i) {
+        return std::min<long long>(streams[i]->counter, streams[i]->window) * streams[i]->n_q;
+    };
+    std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return n_kv(a) > n_kv(b); });
+    auto* p = new (std::nothrow) AttnParams<kMaxBatchStreams>();
+    if (!p) return fail(FRT_ERR_OOM, "host allocation failed");
+    std::memset(p, 0, sizeof(*p));
+    int items = 0;
+    for (int oi = 0; oi < n; ++oi) {
+        const int i = order[oi];
+        frt_stream_t* s = streams[i];
+        AttnStreamDesc& d = p->s[oi];
+        const long long nkv = n_kv(i);
+        if ((st = make_map(&d.q_map, q[i], s->head_dim, s->heads, s->n_q)) != FRT_OK ||
+            (st = make_map(&d.k_map, s->cache_k, s->head_dim, s->heads, nkv)) != FRT_OK ||
+            (st = make_map(&d.v_map, s->cache_v, s->head_dim, s->heads, nkv)) != FRT_OK) {
+            delete p;
+            return st;
+        }
+        d.out = out[i];
+        d.n_q = s->n_q;
+        d.n_kv = int(nkv);
+        d.n_qpairs = (s->n_q + 255) / 256;
+        d.item_begin = items;
+        items += d.n_qpairs * s->heads;
+    }
+    p->n_streams = n;
+    p->heads = s0->heads;
+    p->total_items = items;
+    p->out_bf16 = s0->cfg.out_dtype == FRT_OUT_BF16;
+    p->scale_log2 = float(double(s0->scale) * 1.4426950408889634);
+    p->wait_limit_ns = s0->wait_limit_ns;
+    p->status = s0->status_dev;
+    cudaError_t e = cudaSuccess;
+    for (int i = 1; i < n && e == cudaSuccess; ++i)
+        if (streams[i]->cs != s0->cs) {
+            e = cudaEventRecord(streams[i]->ev, streams[i]->cs);
+            if (e == cudaSuccess) e = cudaStreamWaitEvent(s0->cs, streams[i]->ev, 0);
+        }
+    if (e == cudaSuccess && s0->attn_start) e = cudaEventRecord(s0->attn_start, s0->cs);
+    if (e == cudaSuccess) e = launch_attention_batched(*p, s0->head_dim, s0->cs);
+    if (e == cudaSuccess && s0->attn_stop) e = cudaEventRecord(s0->attn_stop, s0->cs);
+    delete p;
+    if (e != cudaSuccess) return cuda_fail(e, "batched attention launch");
+    bool other = false;
+    for (int i = 1; i < n; ++i) other |= streams[i]->cs != s0->cs;
+    if (other) {
+        if ((e = cudaEventRecord(s0->ev, s0->cs)) != cudaSuccess) return cuda_fail(e, "event");
+        for (int i = 1; i < n; ++i)
+            if (streams[i]->cs != s0->cs &&
+                (e = cudaStreamWaitEvent(streams[i]->cs, s0->ev, 0)) != cudaSuccess)
+                return cuda_fail(e, "event wait");
+    }
+    return FRT_OK;
+}
+
+frt_status frt_stream_sync(frt_stream_t* s) {
+    if (!s) return fail(FRT_ERR_INVALID_ARG, "NULL stream handle");
+    if (!s->configured) return FRT_OK;
+    cudaError_t e = cudaStreamSynchronize(s->cs);
+    if (e != cudaSuccess) return cuda_fail(e, "stream sync");
+    return check_device_status(s);
+}
+
+frt_status frt_stream_reset(frt_stream_t* s) {
+    if (!s) return fail(FRT_ERR_INVALID_ARG, "NULL stream handle");
+    if (!s->configured) return fail(FRT_ERR_STATE, "stream not configured");
+    cudaError_t e = cudaStreamSynchronize(s->cs);
+    if (e != cudaSuccess) return cuda_fail(e, "stream sync");
+    const size_t cache_bytes = size_t(s->window) * s->chunk_elems * 2;
+    if ((e = cudaMemsetAsync(s->cache_k, 0, cache_bytes, s->cs)) != cudaSuccess ||
+        (e = cudaMemsetAsync(s->cache_v, 0, cache_bytes, s->cs)) != cudaSuccess ||
+        (e = cudaStreamSynchronize(s->cs)) != cudaSuccess)
+        return cuda_fail(e, "cache clear");
+    std::memset(s->status_host, 0, sizeof(DeviceStatus));
+    s->counter = 0;
+    s->phase = kStart;
+    s->last_q = s->last_k = s->last_v = nullptr;
+    return FRT_OK;
+}
+
+void frt_stream_destroy(frt_stream_t* s) {
+    if (!s) return;
+    if (s->configured) cudaStreamSynchronize(s->cs);
+    free_device(s);
+    delete s;
+}
+
+long long frt_stream_chunk_counter(const frt_stream_t* s) { return s ? s->counter : -1; }
+
+frt_status frt_stream_set_attention_events(frt_stream_t* s, void* start_event,
+                                           void* stop_event) {
+    if (!s) return fail(FRT_ERR_INVALID_ARG, "NULL stream handle");
+    if ((start_event == nullptr) != (stop_event == nullptr))
+        return fail(FRT_ERR_INVALID_ARG, "give both events or neither");
+    s->attn_start = static_cast<cudaEvent_t>(start_event);
+    s->attn_stop = static_cast<cudaEvent_t>(stop_event);
+    return FRT_OK;
+}
+
+frt_status frt_stream_cache(const frt_stream_t* s, const void** k_cache, const void** v_cache,
+                            long long* rows) {
+    if (!s) return fail(FRT_ERR_INVALID_ARG, "NULL stream handle");
+    if (!s->configured) return fail(FRT_ERR_STATE, "stream not configured");
+    if (k_cache) *k_cache = s->cache_k;
+    if (v_cache) *v_cache = s->cache_v;
+    if (rows) *rows = (long long)s->window * s->n_q;
+    return FRT_OK;
+}
+
+}  // extern "C"
+
+// Device pointer of a stream's status block (used by the self-test entry points).
+extern "C" void* frt_internal_status_dev(frt_stream_t* s) {
+    return (s && s->configured) ? static_cast<void*>(s->status_dev) : nullptr;
+}

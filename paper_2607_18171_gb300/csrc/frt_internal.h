@@ -1,0 +1,123 @@
+// frt_internal.h — parameter blocks shared by the host library and the kernels.
+#pragma once
+#include <stdint.h>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+namespace frt {
+
+// Largest frames_per_chunk * d_t/2 (t-segment cos/sin entries of one chunk, passed by value).
+constexpr int kMaxTEntries = 256;
+// Largest number of streams in one batched attention launch.
+constexpr int kMaxBatchStreams = 32;
+
+// Device status block (host-mapped pinned memory): the first device error wins.
+struct DeviceStatus {
+    int code;      // 0 = ok, else an frt_status value
+    int block;     // blockIdx.x of the CTA that reported it
+    int role;      // 0 producer, 1 mma, 2+ softmax group
+    int where;     // loop iteration or barrier id
+};
+
+// RoPE tables: the t-segment cos/sin of the chunk's F frames (by value) and the
+// per-stream h/w tables (device memory, fp32 from fp64 host computation).
+struct RopeArgs {
+    const float2* hw;   // [grid_h][d_h/2] then [grid_w][d_w/2]
+    int tpf;            // tokens per frame
+    int gh, gw;         // latent grid
+    int dt2, dh2, dw2;  // pairs per segment
+    float2 t_tab[kMaxTEntries];  // [F][d_t/2]
+};
+
+// One pair (x0, x1) packed as bf16x2 (x0 in the low half) turned by (c, s).
+// Every kernel that rotates goes through this routine, so the fused and the
+// separate paths give bit-identical bf16 results.
+__device__ __forceinline__ uint32_t rope_pair(uint32_t x, float c, float s) {
+    const float x0 = __uint_as_float(x << 16);
+    const float x1 = __uint_as_float(x & 0xFFFF0000u);
+    const float y0 = __fmaf_rn(x0, c, __fmul_rn(-x1, s));
+    const float y1 = __fmaf_rn(x0, s, __fmul_rn(x1, c));
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(y1), "f"(y0));
+    return r;
+}
+
+__device__ __forceinline__ float2 rope_cs(const RopeArgs& a, int pi, int f, int r, int col) {
+    if (pi < a.dt2) return a.t_tab[f * a.dt2 + pi];
+    pi -= a.dt2;
+    if (pi < a.dh2) return a.hw[r * a.dh2 + pi];
+    pi -= a.dh2;
+    return a.hw[a.gh * a.dh2 + col * a.dw2 + pi];
+}
+
+// Rotate 8 consecutive head_dim elements [d0, d0+8) (d0 % 8 == 0) of a token at
+// frame f, row r, column col.
+__device__ __forceinline__ uint4 rope_rotate8(uint4 v, int d0, int f, int r, int col,
+                                              const RopeArgs& a) {
+    const int p0 = d0 >> 1;
+    float2 cs;
+    cs = rope_cs(a, p0 + 0, f, r, col); v.x = rope_pair(v.x, cs.x, cs.y);
+    cs = rope_cs(a, p0 + 1, f, r, col); v.y = rope_pair(v.y, cs.x, cs.y);
+    cs = rope_cs(a, p0 + 2, f, r, col); v.z = rope_pair(v.z, cs.x, cs.y);
+    cs = rope_cs(a, p0 + 3, f, r, col); v.w = rope_pair(v.w, cs.x, cs.y);
+    return v;
+}
+
+// ----------------------------------------------------------------------------------------
+// Attention launch parameters
+// ----------------------------------------------------------------------------------------
+struct AttnStreamDesc {
+    CUtensorMap q_map;   // 3D (D, H, Nq), box (64, 1, 128), 128-byte swizzle
+    CUtensorMap k_map;   // 3D (D, H, Nkv), box (64, 1, 128)
+    CUtensorMap v_map;
+    void* out;           // [Nq, H, D] fp32 or bf16
+    int n_q;
+    int n_kv;
+    int n_qpairs;        // ceil(Nq / 256): work items per head
+    int item_begin;      // first work item of this stream
+};
+
+template <int MAXS>
+struct AttnParams {
+    AttnStreamDesc s[MAXS];
+    int n_streams;
+    int heads;
+    int total_items;
+    int out_bf16;
+    float scale_log2;            // sm_scale * log2(e)
+    unsigned long long wait_limit_ns;
+    DeviceStatus* status;
+    RopeArgs rope;               // RoPE-Q prologue (single-stream fused path only)
+};
+
+struct AppendParams {
+    const uint4* k_src;     // [Nq, H, D] bf16
+    const uint4* v_src;
+    uint4* k_dst;           // cache rows of the slot
+    uint4* v_dst;
+    int n_tok;
+    int vec_per_tok;        // H * D / 8
+    int vec_per_head_log2;  // log2(D / 8)
+    int rope;               // rotate K on the way
+    RopeArgs ra;
+};
+
+struct RopeParams {
+    uint4* q;
+    uint4* k;
+    int n_tok;
+    int vec_per_tok;
+    int vec_per_head_log2;
+    RopeArgs ra;
+};
+
+// Kernel launchers (defined in the .cu files).
+cudaError_t launch_rope_qk(const RopeParams& p, cudaStream_t st);
+cudaError_t launch_kv_append(const AppendParams& p, cudaStream_t st);
+cudaError_t launch_attention_single(const AttnParams<1>& p, int head_dim, bool rope_q,
+                                    cudaStream_t st);
+cudaError_t launch_attention_batched(const AttnParams<kMaxBatchStreams>& p, int head_dim,
+                                     cudaStream_t st);
+int num_sms();
+
+}  // namespace frt

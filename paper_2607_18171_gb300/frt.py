@@ -1,0 +1,272 @@
+"""Thin ctypes binding of ``libfrt.so`` (C ABI in ``include/frt.h``).
+
+Argument marshalling only: tensors are passed as raw device pointers and every step
+of the path runs in the library's CUDA kernels. There is no CPU fallback: if the
+library is missing, loading raises.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libfrt.so")
+
+FRT_OK = 0
+STATUS_NAMES = {0: "FRT_OK", 1: "FRT_ERR_INVALID_ARG", 2: "FRT_ERR_STATE", 3: "FRT_ERR_OOM",
+                4: "FRT_ERR_CUDA", 5: "FRT_ERR_UNSUPPORTED", 6: "FRT_ERR_TIMEOUT"}
+OUT_F32, OUT_BF16 = 0, 1
+
+
+class FrtError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {message}")
+        self.status = status
+
+
+class Config(ctypes.Structure):
+    _fields_ = [("grid_h", ctypes.c_int), ("grid_w", ctypes.c_int),
+                ("rope_dt", ctypes.c_int), ("rope_dh", ctypes.c_int), ("rope_dw", ctypes.c_int),
+                ("theta", ctypes.c_double), ("sm_scale", ctypes.c_double),
+                ("out_dtype", ctypes.c_int), ("cuda_stream", ctypes.c_void_p)]
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """Load libfrt.so once and declare its signatures."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is not built; run __graft_entry__.build() "
+                           "(this package has no CPU fallback)")
+    L = ctypes.CDLL(LIB_PATH)
+    P, I, LL, D = ctypes.c_void_p, ctypes.c_int, ctypes.c_longlong, ctypes.c_double
+    sig = {
+        "frt_stream_create": (P, [I, I, I, I, I]),
+        "frt_config_default": (I, [P, ctypes.POINTER(Config)]),
+        "frt_stream_configure": (I, [P, ctypes.POINTER(Config)]),
+        "frt_rope3d_qk": (I, [P, P, P]),
+        "frt_kv_append_evict": (I, [P, P, P, ctypes.POINTER(I), ctypes.POINTER(LL)]),
+        "frt_chunk_attention": (I, [P, P, P, P, P]),
+        "frt_chunk_step": (I, [P, P, P, P, P, ctypes.POINTER(I), ctypes.POINTER(LL)]),
+        "frt_chunk_step_host": (I, [P, P, P, P, P, ctypes.POINTER(I), ctypes.POINTER(LL)]),
+        "frt_chunk_attention_batched": (I, [ctypes.POINTER(P), I, ctypes.POINTER(P),
+                                            ctypes.POINTER(P)]),
+        "frt_stream_sync": (I, [P]),
+        "frt_stream_reset": (I, [P]),
+        "frt_stream_destroy": (None, [P]),
+        "frt_stream_chunk_counter": (LL, [P]),
+        "frt_stream_cache": (I, [P, ctypes.POINTER(P), ctypes.POINTER(P), ctypes.POINTER(LL)]),
+        "frt_stream_set_attention_events": (I, [P, P, P]),
+        "frt_window_index": (I, [LL, I, ctypes.POINTER(I), ctypes.POINTER(LL),
+                                 ctypes.POINTER(I)]),
+        "frt_status_string": (ctypes.c_char_p, [I]),
+        "frt_last_error": (ctypes.c_char_p, []),
+        "frt_version": (ctypes.c_char_p, []),
+        "frt_selftest_umma_tile": (I, [P, P, P, I, I, I, I, P, P]),
+        "frt_selftest_wait_timeout": (I, [P, LL, P]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(L, name)
+        fn.restype = res
+        fn.argtypes = args
+    _ = D
+    _lib = L
+    return L
+
+
+def _check(status: int) -> None:
+    if status != FRT_OK:
+        raise FrtError(status, lib().frt_last_error().decode())
+
+
+def _ptr(t: torch.Tensor | None):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _bf16_dev(t: torch.Tensor, shape, name: str) -> None:
+    if t.dtype != torch.bfloat16 or not t.is_cuda or not t.is_contiguous():
+        raise ValueError(f"{name} must be a contiguous bf16 CUDA tensor")
+    if tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+
+
+def window_index(chunk: int, window: int):
+    """(slot, evicted, valid_chunks) computed by the library (host only)."""
+    s, v = ctypes.c_int(), ctypes.c_int()
+    e = ctypes.c_longlong()
+    _check(lib().frt_window_index(chunk, window, ctypes.byref(s), ctypes.byref(e),
+                                  ctypes.byref(v)))
+    return s.value, e.value, v.value
+
+
+class Stream:
+    """One stream's persistent state (its rolling KV cache) on the current device."""
+
+    def __init__(self, heads: int, head_dim: int, grid_h: int, grid_w: int,
+                 frames_per_chunk: int, window_chunks: int, split=None, theta: float = 10000.0,
+                 sm_scale: float = 0.0, out_dtype: torch.dtype = torch.float32,
+                 cuda_stream: torch.cuda.Stream | None = None):
+        L = lib()
+        self._h = L.frt_stream_create(heads, head_dim, grid_h * grid_w, frames_per_chunk,
+                                      window_chunks)
+        if not self._h:
+            raise FrtError(1, L.frt_last_error().decode())
+        self.heads, self.head_dim = heads, head_dim
+        self.grid_h, self.grid_w = grid_h, grid_w
+        self.frames, self.window = frames_per_chunk, window_chunks
+        self.n_q = frames_per_chunk * grid_h * grid_w
+        self.out_dtype = out_dtype
+        cfg = Config()
+        _check(L.frt_config_default(self._h, ctypes.byref(cfg)))
+        cfg.grid_h, cfg.grid_w = grid_h, grid_w
+        if split is not None:
+            cfg.rope_dt, cfg.rope_dh, cfg.rope_dw = (int(x) for x in split)
+        cfg.theta = theta
+        cfg.sm_scale = sm_scale
+        cfg.out_dtype = OUT_BF16 if out_dtype == torch.bfloat16 else OUT_F32
+        self.torch_stream = cuda_stream or torch.cuda.current_stream()
+        cfg.cuda_stream = ctypes.c_void_p(self.torch_stream.cuda_stream)
+        self.config = cfg
+        _check(L.frt_stream_configure(self._h, ctypes.byref(cfg)))
+
+    # -- lifetime --------------------------------------------------------------------
+    def close(self) -> None:
+        if getattr(self, "_h", None):
+            lib().frt_stream_destroy(self._h)
+            self._h = None
+
+    def __del__(self):  # pragma: no cover - best effort
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    @property
+    def handle(self):
+        return self._h
+
+    @property
+    def counter(self) -> int:
+        return lib().frt_stream_chunk_counter(self._h)
+
+    def shape(self):
+        return (self.n_q, self.heads, self.head_dim)
+
+    def new_out(self) -> torch.Tensor:
+        return torch.empty(self.shape(), dtype=self.out_dtype, device="cuda")
+
+    # -- the three operations ------------------------------------------------------
+    def rope3d_qk(self, q: torch.Tensor, k: torch.Tensor) -> None:
+        _bf16_dev(q, self.shape(), "q"); _bf16_dev(k, self.shape(), "k")
+        _check(lib().frt_rope3d_qk(self._h, _ptr(q), _ptr(k)))
+
+    def kv_append_evict(self, k: torch.Tensor, v: torch.Tensor):
+        _bf16_dev(k, self.shape(), "k"); _bf16_dev(v, self.shape(), "v")
+        slot, ev = ctypes.c_int(), ctypes.c_longlong()
+        _check(lib().frt_kv_append_evict(self._h, _ptr(k), _ptr(v), ctypes.byref(slot),
+                                         ctypes.byref(ev)))
+        return slot.value, ev.value
+
+    def chunk_attention(self, q: torch.Tensor, out: torch.Tensor, k=None, v=None) -> None:
+        _bf16_dev(q, self.shape(), "q")
+        self._check_out(out)
+        _check(lib().frt_chunk_attention(_ptr(q), _ptr(k), _ptr(v), _ptr(out), self._h))
+
+    def chunk_step(self, q, k, v, out):
+        for t, n in ((q, "q"), (k, "k"), (v, "v")):
+            _bf16_dev(t, self.shape(), n)
+        self._check_out(out)
+        slot, ev = ctypes.c_int(), ctypes.c_longlong()
+        _check(lib().frt_chunk_step(self._h, _ptr(q), _ptr(k), _ptr(v), _ptr(out),
+                                    ctypes.byref(slot), ctypes.byref(ev)))
+        return slot.value, ev.value
+
+    def chunk_step_host(self, q_host, k_host, v_host, out_host):
+        """Host tensors in, host tensor out (copies enqueued on the stream)."""
+        for t in (q_host, k_host, v_host, out_host):
+            if t.is_cuda or not t.is_contiguous():
+                raise ValueError("host buffers must be contiguous CPU tensors")
+        slot, ev = ctypes.c_int(), ctypes.c_longlong()
+        _check(lib().frt_chunk_step_host(self._h, _ptr(q_host), _ptr(k_host), _ptr(v_host),
+                                         _ptr(out_host), ctypes.byref(slot), ctypes.byref(ev)))
+        return slot.value, ev.value
+
+    def sync(self) -> None:
+        _check(lib().frt_stream_sync(self._h))
+
+    def reset(self) -> None:
+        _check(lib().frt_stream_reset(self._h))
+
+    def set_attention_events(self, start: torch.cuda.Event | None,
+                             stop: torch.cuda.Event | None) -> None:
+        """Record these events around every attention kernel launch of this stream."""
+        _check(lib().frt_stream_set_attention_events(
+            self._h, None if start is None else ctypes.c_void_p(start.cuda_event),
+            None if stop is None else ctypes.c_void_p(stop.cuda_event)))
+
+    def cache(self):
+        """(k_cache, v_cache) device tensors viewing the stream's ring buffer
+        [W * Nq, heads, head_dim] bf16 (read-only use)."""
+        kp, vp = ctypes.c_void_p(), ctypes.c_void_p()
+        rows = ctypes.c_longlong()
+        _check(lib().frt_stream_cache(self._h, ctypes.byref(kp), ctypes.byref(vp),
+                                      ctypes.byref(rows)))
+        return (_view_bf16(kp.value, (rows.value, self.heads, self.head_dim)),
+                _view_bf16(vp.value, (rows.value, self.heads, self.head_dim)))
+
+    def _check_out(self, out):
+        if out.dtype != self.out_dtype or not out.is_cuda or not out.is_contiguous() or \
+                tuple(out.shape) != self.shape():
+            raise ValueError("out must be a contiguous CUDA tensor of the stream's out dtype/shape")
+
+
+def _view_bf16(ptr: int, shape) -> torch.Tensor:
+    """Non-owning torch view of library-owned device memory."""
+    n = 1
+    for s in shape:
+        n *= s
+
+    class _Holder:
+        __cuda_array_interface__ = {"shape": (n,), "typestr": "<u2", "data": (ptr, False),
+                                    "version": 3, "strides": None}
+
+    t = torch.as_tensor(_Holder(), device="cuda")
+    return t.view(torch.bfloat16).view(*shape)
+
+
+def chunk_attention_batched(streams, qs, outs) -> None:
+    n = len(streams)
+    for s, q, o in zip(streams, qs, outs):
+        _bf16_dev(q, s.shape(), "q")
+        s._check_out(o)
+    arr = ctypes.c_void_p * n
+    _check(lib().frt_chunk_attention_batched(
+        arr(*[s.handle for s in streams]), n, arr(*[q.data_ptr() for q in qs]),
+        arr(*[o.data_ptr() for o in outs])))
+
+
+def selftest_umma_tile(a: torch.Tensor, b: torch.Tensor, b_mn_major: bool, lbo: int = 16384,
+                       sbo: int = 1024, a_from_tmem: bool = False) -> torch.Tensor:
+    c = torch.empty(128, 128, dtype=torch.float32, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    rc = lib().frt_selftest_umma_tile(_ptr(a), _ptr(b), _ptr(c), int(b_mn_major), lbo, sbo,
+                                      int(a_from_tmem), _ptr(status),
+                                      ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+    if rc != 0:
+        raise FrtError(4, f"selftest launch failed ({rc})")
+    torch.cuda.synchronize()
+    if int(status.item()) != 0:
+        raise FrtError(6, "selftest tile timed out")
+    return c
+
+
+def selftest_wait_timeout(stream: Stream, limit_ns: int) -> None:
+    _check(lib().frt_selftest_wait_timeout(
+        stream.handle, limit_ns, ctypes.c_void_p(stream.torch_stream.cuda_stream)))

@@ -1,0 +1,116 @@
+"""C ABI checks that need no GPU: the library builds and loads, exports every symbol
+the headers declare, host-side window arithmetic is exact, and argument/state
+validation rejects bad calls before any device work."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def frt():
+    from paper_2607_18171_gb300 import _build, frt as m
+    _build.build()
+    m.lib()
+    return m
+
+
+def declared_symbols():
+    names = set()
+    for h in ("frt.h", "frt_selftest.h"):
+        src = open(os.path.join(ROOT, "include", h)).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        names.update(re.findall(r"\b(frt_[a-z0-9_]+)\s*\(", src))
+    return names
+
+
+def test_library_exports_every_declared_symbol(frt):
+    L = frt.lib()
+    names = declared_symbols()
+    assert {"frt_stream_create", "frt_rope3d_qk", "frt_kv_append_evict",
+            "frt_chunk_attention"} <= names
+    for n in names:
+        assert hasattr(L, n), n
+
+
+@pytest.mark.parametrize("window", [1, 2, 3, 7])
+def test_window_index_bit_exact(frt, window):
+    for c in list(range(0, 51)) + [2**31 + 5, 2**40 + 3]:
+        slot, ev, valid = frt.window_index(c, window)
+        assert slot == c % window
+        assert ev == (c - window if c >= window else -1)
+        assert valid == min(c + 1, window)
+
+
+def test_window_index_rejects_bad_args(frt):
+    with pytest.raises(frt.FrtError) as e:
+        frt.window_index(-1, 3)
+    assert e.value.status == 1
+    with pytest.raises(frt.FrtError):
+        frt.window_index(0, 0)
+
+
+def test_status_strings(frt):
+    L = frt.lib()
+    for code, name in frt.STATUS_NAMES.items():
+        assert L.frt_status_string(code).decode() == name
+
+
+def test_create_validates_shapes(frt):
+    L = frt.lib()
+    assert not L.frt_stream_create(2, 96, 16, 3, 3)
+    assert "head_dim" in L.frt_last_error().decode()
+    assert not L.frt_stream_create(0, 64, 16, 3, 3)
+    assert not L.frt_stream_create(2, 64, 16, 3, 0)
+    assert not L.frt_stream_create(2, 64, 1 << 20, 3, 3)
+    h = L.frt_stream_create(2, 64, 16, 3, 3)
+    assert h
+    L.frt_stream_destroy(h)
+
+
+def test_configure_rejects_bad_config_before_device_work(frt):
+    L = frt.lib()
+    h = L.frt_stream_create(2, 64, 16, 3, 3)
+    cfg = frt.Config()
+    assert L.frt_config_default(h, ctypes.byref(cfg)) == 0
+    assert (cfg.rope_dt, cfg.rope_dh, cfg.rope_dw) == (16, 24, 24)
+    assert abs(cfg.sm_scale - 0.125) < 1e-15 and cfg.theta == 10000.0
+    bad = frt.Config.from_buffer_copy(cfg)
+    bad.grid_h, bad.grid_w = 3, 5          # 15 != 16 tokens per frame
+    assert L.frt_stream_configure(h, ctypes.byref(bad)) == 1
+    bad = frt.Config.from_buffer_copy(cfg)
+    bad.grid_h, bad.grid_w = 4, 4
+    bad.rope_dt, bad.rope_dh, bad.rope_dw = 15, 25, 24  # odd
+    assert L.frt_stream_configure(h, ctypes.byref(bad)) == 1
+    bad.rope_dt, bad.rope_dh, bad.rope_dw = 16, 24, 26  # sum != 64
+    assert L.frt_stream_configure(h, ctypes.byref(bad)) == 1
+    L.frt_stream_destroy(h)
+
+
+def test_calls_before_configure_are_state_errors(frt):
+    L = frt.lib()
+    h = L.frt_stream_create(2, 64, 16, 3, 3)
+    buf = ctypes.create_string_buffer(64)
+    p = ctypes.cast(buf, ctypes.c_void_p)
+    assert L.frt_rope3d_qk(h, p, p) == 2
+    assert L.frt_kv_append_evict(h, p, p, None, None) == 2
+    assert L.frt_chunk_attention(p, None, None, p, h) == 2
+    assert L.frt_chunk_step(h, p, p, p, p, None, None) == 2
+    assert L.frt_stream_reset(h) == 2
+    assert L.frt_stream_chunk_counter(h) == 0
+    assert L.frt_rope3d_qk(None, p, p) == 1
+    L.frt_stream_destroy(h)
+    L.frt_stream_destroy(None)
+
+
+def test_product_path_does_not_import_the_oracle():
+    pkg = os.path.join(ROOT, "paper_2607_18171_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            if f.endswith(".py"):
+                src = open(os.path.join(dirpath, f)).read()
+                assert not re.search(r"^\s*(import|from)\s+oracle", src, flags=re.M), f

@@ -1,0 +1,152 @@
+"""GPU vs fp64 oracle on sizes the oracle finishes in seconds: every output element,
+several tiles, ragged tails; fused vs separate paths; determinism; indices."""
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2607_18171_gb300 import synth
+from tests import parity_util as U
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def frt():
+    from paper_2607_18171_gb300 import frt as m
+    m.lib()
+    return m
+
+
+SMALL = {
+    # ragged: Nq = 3*130 = 390 (second 256-row item has one partial tile), Nkv up to 1170
+    "ragged_d128": synth.Workload("ragged_d128", 90, 1, 3, 128, 10, 13, 3, 3, 5, (32, 48, 48)),
+    # one frame per chunk, Nq = 7*19 = 133 (tile 2 holds 5 rows), window 4, per-head scales
+    "ragged_scaled": synth.Workload("ragged_scaled", 91, 1, 2, 128, 7, 19, 1, 4, 6, (32, 48, 48),
+                                    head_scale=True),
+    # head_dim 64 beyond one KV tile: Nq = 2*80 = 160, window 2 -> Nkv 320
+    "d64_multi_tile": synth.Workload("d64_multi_tile", 92, 1, 3, 64, 8, 10, 2, 2, 4, (16, 24, 24)),
+    # window 1: plain bidirectional attention per chunk
+    "window1": synth.Workload("window1", 93, 1, 2, 128, 5, 9, 2, 1, 3, (32, 48, 48)),
+}
+
+
+@pytest.mark.parametrize("name", ["tiny"] + list(SMALL))
+@pytest.mark.parametrize("fused", [True, False])
+def test_stream_matches_oracle_every_element(frt, name, fused):
+    wl = synth.WORKLOADS.get(name) or SMALL[name]
+    st = U.make_stream(wl, frt)
+    run = U.run_fused if fused else U.run_separate
+    got = run(st, wl, 0, wl.chunks, keep=range(wl.chunks))
+    ref = U.oracle_full_stream(wl, 0, wl.chunks)
+    for c in range(wl.chunks):
+        out, slot, ev = got[c]
+        r_out, r_slot, r_ev = ref[c]
+        assert (slot, ev) == (r_slot, r_ev)
+        U.assert_close(out, r_out, f"{name} chunk {c}")
+    st.close()
+
+
+@pytest.mark.parametrize("name", ["tiny", "ragged_d128"])
+def test_fused_and_separate_paths_are_bit_identical(frt, name):
+    wl = synth.WORKLOADS.get(name) or SMALL[name]
+    a = U.make_stream(wl, frt)
+    b = U.make_stream(wl, frt)
+    ra = U.run_fused(a, wl, 0, wl.chunks, keep=range(wl.chunks))
+    rb = U.run_separate(b, wl, 0, wl.chunks, keep=range(wl.chunks))
+    for c in range(wl.chunks):
+        assert np.array_equal(ra[c][0], rb[c][0]), f"chunk {c}"
+    ka, va = a.cache()
+    kb, vb = b.cache()
+    assert torch.equal(ka.view(torch.int16), kb.view(torch.int16))
+    assert torch.equal(va.view(torch.int16), vb.view(torch.int16))
+    a.close(); b.close()
+
+
+def test_run_to_run_determinism(frt):
+    wl = SMALL["ragged_d128"]
+    outs = []
+    for _ in range(2):
+        st = U.make_stream(wl, frt)
+        outs.append(U.run_fused(st, wl, 0, wl.chunks, keep=range(wl.chunks)))
+        st.close()
+    for c in range(wl.chunks):
+        assert np.array_equal(outs[0][c][0], outs[1][c][0])
+
+
+def test_bf16_output(frt):
+    wl = SMALL["ragged_d128"]
+    st = U.make_stream(wl, frt, out_dtype=torch.bfloat16)
+    got = U.run_fused(st, wl, 0, wl.chunks, keep=range(wl.chunks))
+    ref = U.oracle_full_stream(wl, 0, wl.chunks)
+    for c in range(wl.chunks):
+        U.assert_close(got[c][0], ref[c][0], f"bf16 chunk {c}")
+    st.close()
+
+
+def test_rope_within_one_bf16_ulp_of_oracle(frt):
+    from oracle.frt_oracle import bf16_round, rope3d
+    wl = SMALL["ragged_d128"]
+    st = U.make_stream(wl, frt)
+    for c in range(3):
+        q, k, v = synth.chunk_qkv(wl, 0, c)
+        qd, kd = q.cuda(), k.cuda()
+        st.rope3d_qk(qd, kd)
+        st.kv_append_evict(kd, v.cuda())
+        args = (c, wl.grid_h, wl.grid_w, wl.frames, wl.split)
+        for got, src in ((qd, q), (kd, k)):
+            ref = bf16_round(rope3d(synth.as_f64(src), *args))
+            g = got.float().cpu().numpy().astype(np.float64)
+            ulp = np.ldexp(1.0, np.frexp(np.maximum(np.abs(ref), 1e-30))[1] - 8)
+            dev = np.abs(g - ref) / ulp
+            assert dev.max() <= 1.0, dev.max()
+            assert (dev == 0).mean() > 0.99
+    st.close()
+
+
+def test_append_writes_slot_bytes_and_evicts_whole_chunks(frt):
+    wl = SMALL["ragged_d128"]
+    st = U.make_stream(wl, frt)
+    kept = {}
+    for c in range(7):
+        q, k, v = U.gpu_inputs(wl, 0, c)
+        st.rope3d_qk(q, k)
+        slot, ev = st.kv_append_evict(k, v)
+        assert slot == c % wl.window and ev == (c - wl.window if c >= wl.window else -1)
+        kept[c] = (k.clone(), v.clone())
+    st.sync()
+    kc, vc = st.cache()
+    nq = wl.n_q
+    for c in range(7 - wl.window, 7):
+        s = c % wl.window
+        assert torch.equal(kc[s * nq:(s + 1) * nq].view(torch.int16), kept[c][0].view(torch.int16))
+        assert torch.equal(vc[s * nq:(s + 1) * nq].view(torch.int16), kept[c][1].view(torch.int16))
+    st.close()
+
+
+def test_batched_ragged_streams_match_single_launches_and_oracle(frt):
+    base = SMALL["ragged_d128"]
+    fills = [3, 1, 2, 3]
+    streams, outs_b, outs_s, qs = [], [], [], []
+    for s, fill in enumerate(fills):
+        st = U.make_stream(base, frt)
+        for c in range(fill - 1):
+            q, k, v = U.gpu_inputs(base, s, c)
+            st.chunk_step(q, k, v, st.new_out())
+        q, k, v = U.gpu_inputs(base, s, fill - 1)
+        st.rope3d_qk(q, k)
+        st.kv_append_evict(k, v)
+        streams.append(st); qs.append(q)
+        outs_b.append(st.new_out())
+    frt.chunk_attention_batched(streams, qs, outs_b)
+    for st, q in zip(streams, qs):
+        o = st.new_out()
+        st.chunk_attention(q, o)
+        outs_s.append(o)
+    torch.cuda.synchronize()
+    for s, fill in enumerate(fills):
+        assert torch.equal(outs_b[s], outs_s[s]), s
+        ref = U.oracle_full_stream(base, s, fill)[fill - 1][0]
+        U.assert_close(outs_b[s].cpu().numpy(), ref, f"stream {s}")
+    for st in streams:
+        st.close()
