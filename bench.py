@@ -118,6 +118,19 @@ class ClockSampler:
                 "samples": len(sm), "reasons": sorted(reasons)}
 
 
+def timing_events(n, stream):
+    """n (start, stop) CUDA event pairs, recorded once so that the driver-level events
+    exist before their handles are handed to the library."""
+    import torch
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(n)]
+    for a, b in evs:
+        a.record(stream)
+        b.record(stream)
+    torch.cuda.synchronize()
+    return evs
+
+
 def init_dist():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -175,8 +188,7 @@ def run_gpu(args, wl, world, rank, local):
         step(i)
     st.sync()
     n = args.steps
-    ev_a = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-            for _ in range(n)]
+    ev_a = timing_events(n, stream)
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     if world > 1:
         torch.distributed.barrier()
@@ -288,8 +300,7 @@ def run_gpu_multi(args, wl, world, rank, local, dev, peak_tf, peak_kind):
         step(i)
     torch.cuda.synchronize()
     n = args.steps
-    ev_a = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-            for _ in range(n)]
+    ev_a = timing_events(n, stream)
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     if world > 1:
         torch.distributed.barrier()

@@ -95,12 +95,16 @@ def test_rope_within_one_bf16_ulp_of_oracle(frt):
         st.kv_append_evict(kd, v.cuda())
         args = (c, wl.grid_h, wl.grid_w, wl.frames, wl.split)
         for got, src in ((qd, q), (kd, k)):
-            ref = bf16_round(rope3d(synth.as_f64(src), *args))
+            x = synth.as_f64(src)
+            ref = bf16_round(rope3d(x, *args))
             g = got.float().cpu().numpy().astype(np.float64)
             ulp = np.ldexp(1.0, np.frexp(np.maximum(np.abs(ref), 1e-30))[1] - 8)
-            dev = np.abs(g - ref) / ulp
-            assert dev.max() <= 1.0, dev.max()
-            assert (dev == 0).mean() > 0.99
+            # fp32 rotation with fp32 cos/sin: absolute error <= ~3 * 2^-24 * |pair|,
+            # which exceeds one bf16 ulp of the result only under cancellation
+            pair = np.sqrt(x[..., 0::2] ** 2 + x[..., 1::2] ** 2).repeat(2, axis=-1)
+            bound = ulp + 2.0**-21 * pair
+            assert np.all(np.abs(g - ref) <= bound), float(np.max(np.abs(g - ref) / bound))
+            assert np.mean(g == ref) > 0.99
     st.close()
 
 

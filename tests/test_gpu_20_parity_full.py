@@ -63,8 +63,9 @@ def test_multi_stream_batched_sampled_rows(frt):
 
 
 def test_full_size_whole_output_properties(frt):
-    """Any size: a chunk whose V is constant per head gives that constant everywhere
-    (softmax weights sum to 1), and outputs stay inside the convex hull of V."""
+    """Any size: a chunk whose V is constant per head gives that constant everywhere,
+    because the softmax weights sum to 1 -- up to the bf16 rounding of P in the PV
+    product (each weight within a relative 2^-9, so the sum within 2^-8)."""
     wl = synth.WORKLOADS["dit1p3b"]
     st = U.make_stream(wl, frt)
     const = torch.linspace(-2, 2, wl.heads)
@@ -75,5 +76,5 @@ def test_full_size_whole_output_properties(frt):
         st.chunk_step(q, k, v.contiguous().cuda(), out)
     st.sync()
     ref = const.to(torch.bfloat16).float().view(1, -1, 1)
-    assert (out.cpu() - ref).abs().max().item() < 1e-5
+    assert ((out.cpu() - ref).abs() <= 2.0**-8 * ref.abs() + 1e-6).all()
     st.close()
