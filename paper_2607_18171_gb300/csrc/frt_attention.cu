@@ -5,19 +5,26 @@
 // chunk, all earlier chunks of the window), bf16 operands, fp32 accumulation.
 //
 // One CTA = one work item = (stream, head, 256 query rows as two 128-row tiles).
-// Warp roles (320 threads, one CTA per SM):
-//   warp 0      TMA producer: Q tiles once, then K/V tiles through a STAGES-deep ring
-//               in the order the MMA consumes them (K0, K1, V0, K2, V1, ...).
+// Three warpgroups (384 threads, one CTA per SM); registers are rebalanced with
+// setmaxnreg: warpgroup 0 drops to kRegsCtl, the two softmax warpgroups rise to kRegsSm.
+//   warp 0      TMA producer: Q tiles once, then K/V tiles (K0, V0, K1, V1, ...) through
+//               a STAGES-deep shared-memory ring.
 //   warp 1      TMEM allocator + single-thread tcgen05.mma issuer:
-//                 S_g = Q_g K_j^T  (M=128, N=128, K=D; fp32 in TMEM)
-//                 O_g += P_g V_j   (M=128, N=D,   K=128; fp32 in TMEM)
-//   warps 2-5   softmax group 0 (query tile 0), one thread per query row
-//   warps 6-9   softmax group 1 (query tile 1)
+//                 S_g  = Q_g K_j^T  A, B from shared memory (K-major, 128-byte swizzle)
+//                 O_g += P_g V_j    A = P from TMEM, B = V from shared memory (MN-major)
+//               issued as PV_0(j), S_0(j+1), PV_1(j), S_1(j+1): the tiles alternate
+//   warps 2-3   idle
+//   warps 4-7   softmax group 0 (query tile 0), one thread per query row
+//   warps 8-11  softmax group 1 (query tile 1)
 // TMEM (512 columns): S_0 [0,128), S_1 [128,256), O_0 [256,256+D), O_1 [256+D,256+2D).
-// The softmax threads read S with tcgen05.ld, keep a running max in the log2 domain,
-// write P (bf16) to shared memory in the 128-byte-swizzled K-major layout the MMA
-// reads, and rescale O in TMEM only when the running max grows by more than
-// 2^kRescaleLog2 (O and the row sum stay consistently scaled, so the result is exact).
+// P_g (bf16 pairs) overwrites the first 64 columns of S_g once the scores are in
+// registers. PV_g(j) is issued before S_g(j+1); tcgen05.mma from one thread executes
+// in issue order, so S_g(j+1) never overwrites P_g(j) early, and the arrival of S_g(j)
+// implies PV_g(j-1) is complete (so O_g may be rescaled then). While one tile's softmax
+// runs, the tensor pipe works on the other tile's PV and next S.
+// The softmax keeps a running max in the log2 domain and rescales O only when the row
+// max grows by more than 2^kRescaleLog2 (O and the row sum share the stale max, so the
+// result is exact).
 //
 // Every wait is bounded (mbar_wait): a role that gives up records FRT_ERR_TIMEOUT in the
 // stream's status block, raises a CTA-wide abort flag, and the CTA drains its in-flight
@@ -29,7 +36,13 @@ namespace frt {
 
 namespace {
 
-constexpr int kThreads = 320;
+constexpr int kThreads = 384;
+// Register split: 128 threads x kRegsCtl + 256 threads x kRegsSm must equal the launch
+// allocation 384 x kRegsLaunch (checked on the host before every first launch).
+constexpr int kRegsLaunch = 168;
+constexpr int kRegsCtl = 104;
+constexpr int kRegsSm = 200;
+static_assert(128 * kRegsCtl + 256 * kRegsSm == kThreads * kRegsLaunch, "register split");
 constexpr int kBM = 128;   // query rows per tile
 constexpr int kBN = 128;   // KV rows per tile
 constexpr float kRescaleLog2 = 8.0f;
@@ -40,11 +53,9 @@ struct Cfg {
     static constexpr int NCB = D / 64;                 // 128-byte column blocks per row
     static constexpr int Q_TILE = kBM * D * 2;
     static constexpr int KV_TILE = kBN * D * 2;
-    static constexpr int P_TILE = kBM * kBN * 2;
-    static constexpr int STAGES = (D == 128) ? 3 : 6;
+    static constexpr int STAGES = (D == 128) ? 5 : 8;
     static constexpr int OFF_Q = 0;
-    static constexpr int OFF_P = OFF_Q + 2 * Q_TILE;
-    static constexpr int OFF_KV = OFF_P + 2 * P_TILE;
+    static constexpr int OFF_KV = OFF_Q + 2 * Q_TILE;
     static constexpr int OFF_BAR = OFF_KV + STAGES * KV_TILE;
     static constexpr int SMEM = OFF_BAR + 256 + 1024;  // barriers + alignment slack
     static constexpr uint32_t IDESC_S = idesc_bf16_f32(kBM, kBN, false);
@@ -55,10 +66,9 @@ struct Bars {
     uint64_t q_full;
     uint64_t q_ready[2];
     uint64_t s_full[2];
-    uint64_t s_free[2];
     uint64_t p_full[2];
     uint64_t o_done[2];
-    uint64_t drain;
+    uint64_t drain[2];
     uint64_t kv_full[8];
     uint64_t kv_empty[8];
     uint32_t tmem_base;
@@ -79,20 +89,6 @@ __device__ __forceinline__ void report(DeviceStatus* st, volatile int* abort, in
     }
 }
 
-// Position of KV load number L in the consumption order K0, K1, V0, K2, V1, ...
-// Returns the tile index and whether it is a V tile.
-__device__ __forceinline__ void kv_load_at(int L, int n_tiles, int& tile, bool& is_v) {
-    if (L == 0) { tile = 0; is_v = false; return; }
-    // after K0: pairs (K_{t}, V_{t-1}) for t = 1..n-1, then V_{n-1}
-    const int t = (L + 1) >> 1;            // L=1 -> t=1 (K1), L=2 -> t=1 (V0) ...
-    if (t < n_tiles) {
-        if (L & 1) { tile = t; is_v = false; }
-        else       { tile = t - 1; is_v = true; }
-    } else {
-        tile = n_tiles - 1; is_v = true;   // L = 2n-1
-    }
-}
-
 template <int D, int MAXS, bool ROPE>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
@@ -102,7 +98,6 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                                                ~uintptr_t(1023));
     Bars* bars = reinterpret_cast<Bars*>(smem + C::OFF_BAR);
     const uint32_t sQ = smem_u32(smem + C::OFF_Q);
-    const uint32_t sP = smem_u32(smem + C::OFF_P);
     const uint32_t sKV = smem_u32(smem + C::OFF_KV);
     volatile int* abort = &bars->abort_flag;
 
@@ -115,6 +110,7 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
     const int head = local / sd.n_qpairs;
     const int m0 = (local - head * sd.n_qpairs) * (2 * kBM);
     const bool active1 = (m0 + kBM) < sd.n_q;
+    const int ng = active1 ? 2 : 1;
     const int n_tiles = (sd.n_kv + kBN - 1) / kBN;
     const int n_loads = 2 * n_tiles;
 
@@ -126,11 +122,11 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
         for (int g = 0; g < 2; ++g) {
             mbar_init(smem_u32(&bars->q_ready[g]), kBM);
             mbar_init(smem_u32(&bars->s_full[g]), 1);
-            mbar_init(smem_u32(&bars->s_free[g]), kBM);
             mbar_init(smem_u32(&bars->p_full[g]), kBM);
             mbar_init(smem_u32(&bars->o_done[g]), 1);
         }
-        mbar_init(smem_u32(&bars->drain), 1);
+        mbar_init(smem_u32(&bars->drain[0]), 1);
+        mbar_init(smem_u32(&bars->drain[1]), 1);
         for (int s = 0; s < C::STAGES; ++s) {
             mbar_init(smem_u32(&bars->kv_full[s]), 1);
             mbar_init(smem_u32(&bars->kv_empty[s]), 1);
@@ -149,15 +145,17 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
     const uint32_t tmem = bars->tmem_base;
     const uint64_t lim = p.wait_limit_ns;
 
-    if (warp == 0) {
+    if (warp < 4) {
+      asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsCtl));
+      if (warp == 0) {
         // ================================ TMA producer =================================
         if (lane == 0) {
             tma_prefetch_map(&sd.q_map);
             tma_prefetch_map(&sd.k_map);
             tma_prefetch_map(&sd.v_map);
             const uint32_t qbar = smem_u32(&bars->q_full);
-            mbar_arrive_expect_tx(qbar, (active1 ? 2 : 1) * C::Q_TILE);
-            for (int g = 0; g < (active1 ? 2 : 1); ++g)
+            mbar_arrive_expect_tx(qbar, ng * C::Q_TILE);
+            for (int g = 0; g < ng; ++g)
                 for (int cb = 0; cb < C::NCB; ++cb)
                     tma_load_3d(sQ + g * C::Q_TILE + cb * (kBM * 128), &sd.q_map, qbar,
                                 cb * 64, head, m0 + g * kBM);
@@ -170,14 +168,13 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                     report(p.status, abort, 0, L);
                     break;
                 }
-                int tile; bool is_v;
-                kv_load_at(L, n_tiles, tile, is_v);
-                const CUtensorMap* map = is_v ? &sd.v_map : &sd.k_map;
+                const CUtensorMap* map = (L & 1) ? &sd.v_map : &sd.k_map;
+                const int row = (L >> 1) * kBN;
                 const uint32_t fb = smem_u32(&bars->kv_full[stage]);
                 mbar_arrive_expect_tx(fb, C::KV_TILE);
                 const uint32_t dst = sKV + stage * C::KV_TILE;
                 for (int cb = 0; cb < C::NCB; ++cb)
-                    tma_load_3d(dst + cb * (kBN * 128), map, fb, cb * 64, head, tile * kBN);
+                    tma_load_3d(dst + cb * (kBN * 128), map, fb, cb * 64, head, row);
             }
             // drain: every issued load must have landed before the CTA may exit
             const int first = (L - C::STAGES) > 0 ? (L - C::STAGES) : 0;
@@ -186,18 +183,23 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                           lim, abort);
             mbar_wait(qbar, 0, lim, abort);
         }
-    } else if (warp == 1) {
-        // ================================ MMA issuer ===================================
+      } else if (warp == 1) {
+        // ============ MMA issuer: one thread, tiles alternate on the tensor pipe ============
         if (lane == 0) {
             bool ok = true;
-            const int ng = active1 ? 2 : 1;
             for (int g = 0; g < ng && ok; ++g)
                 if (!mbar_wait(smem_u32(&bars->q_ready[g]), 0, lim, abort)) {
                     report(p.status, abort, 1, -1 - g);
                     ok = false;
                 }
             tc_fence_after();
-            int L = 0;
+            // tcgen05.mma issue blocks until the tensor pipe has (nearly) drained the
+            // previous MMA, so every instruction between MMAs is tensor idle time: the
+            // descriptors are precomputed and advanced by constant adds (a descriptor is
+            // linear in its 16-byte start address; addresses stay below 256 KB, no carry).
+            const uint64_t dq0 = sdesc_sw128(sQ, 16, 1024);
+            const uint64_t dk0 = sdesc_sw128(sKV, 16, 1024);
+            const uint64_t dv0 = sdesc_sw128(sKV, kBN * 128, 1024);
             auto wait_load = [&](int Lw) -> bool {
                 if (!mbar_wait(smem_u32(&bars->kv_full[Lw % C::STAGES]), (Lw / C::STAGES) & 1,
                                lim, abort)) {
@@ -207,78 +209,87 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 tc_fence_after();
                 return true;
             };
-            auto issue_s = [&](int g, int stage) {
+            // MMA groups: S_g = Q_g K^T (8 MMAs over D) and O_g += P_g V (8 MMAs over the
+            // KV tile). `mid` runs after the first MMA of a group, while the tensor pipe
+            // still has work queued: waits for loads needed later are hidden there.
+            auto issue_s = [&](int g, int stage, auto&& mid) {
+                const uint64_t dq = dq0 + uint64_t((g * C::Q_TILE) >> 4);
+                const uint64_t dk = dk0 + uint64_t((stage * C::KV_TILE) >> 4);
                 const uint32_t d = tmem + g * kBN;
-                const uint32_t qa = sQ + g * C::Q_TILE;
-                const uint32_t kb = sKV + stage * C::KV_TILE;
 #pragma unroll
                 for (int k = 0; k < D / 16; ++k) {
-                    const uint32_t off = (k >> 2) * (kBM * 128) + (k & 3) * 32;
-                    umma_ss(d, sdesc_sw128(qa + off, 16, 1024), sdesc_sw128(kb + off, 16, 1024),
-                            C::IDESC_S, k > 0 ? 1u : 0u);
+                    const uint64_t off = uint64_t((k >> 2) * ((kBM * 128) >> 4) + (k & 3) * 2);
+                    umma_ss(d, dq + off, dk + off, C::IDESC_S, k > 0 ? 1u : 0u);
+                    if (k == 0) mid();
                 }
                 umma_commit(smem_u32(&bars->s_full[g]));
             };
-            auto issue_o = [&](int g, int stage, bool acc) {
+            auto issue_o = [&](int g, int stage, bool acc, auto&& mid) {
+                const uint64_t dv = dv0 + uint64_t((stage * C::KV_TILE) >> 4);
                 const uint32_t d = tmem + 256 + g * D;
-                const uint32_t pa = sP + g * C::P_TILE;
-                const uint32_t vb = sKV + stage * C::KV_TILE;
+                const uint32_t pa = tmem + g * kBN;   // P_g: bf16 pairs in S_g's columns
 #pragma unroll
                 for (int k = 0; k < kBN / 16; ++k) {
-                    const uint32_t aoff = (k >> 2) * (kBM * 128) + (k & 3) * 32;
-                    const uint32_t boff = k * (16 * 128);
-                    umma_ss(d, sdesc_sw128(pa + aoff, 16, 1024),
-                            sdesc_sw128(vb + boff, kBN * 128, 1024), C::IDESC_O,
+                    umma_ts(d, pa + k * 8, dv + uint64_t(k * ((16 * 128) >> 4)), C::IDESC_O,
                             (acc || k > 0) ? 1u : 0u);
+                    if (k == 0) mid();
                 }
-                umma_commit(smem_u32(&bars->o_done[g]));
             };
-            if (ok && (ok = wait_load(L))) {
-                const int k0 = L % C::STAGES;
-                for (int g = 0; g < ng; ++g) issue_s(g, k0);
-                umma_commit(smem_u32(&bars->kv_empty[k0]));
-                ++L;
+            auto wait_p = [&](int g, int j) -> bool {
+                if (!mbar_wait(smem_u32(&bars->p_full[g]), j & 1, lim, abort)) {
+                    report(p.status, abort, 1, 2000 + j);
+                    return false;
+                }
+                tc_fence_after();
+                return true;
+            };
+            auto nop = [] {};
+            // load order of the producer: K0, V0, K1, V1, ... -> load 2j is K_j, 2j+1 is V_j
+            if (ok && (ok = wait_load(0))) {
+                issue_s(0, 0, nop);
+                if (ng == 2) issue_s(1, 0, [&] { ok = wait_load(1); });
+                else ok = wait_load(1);
+                umma_commit(smem_u32(&bars->kv_empty[0]));
             }
             for (int j = 0; j < n_tiles && ok; ++j) {
                 const bool more = (j + 1) < n_tiles;
-                int kst = -1, vst;
-                if (more) {
-                    if (!(ok = wait_load(L))) break;
-                    kst = L % C::STAGES;
-                    ++L;
-                }
-                if (!(ok = wait_load(L))) break;
-                vst = L % C::STAGES;
-                ++L;
-                for (int g = 0; g < ng && ok; ++g) {
-                    if (more) {
-                        if (!mbar_wait(smem_u32(&bars->s_free[g]), j & 1, lim, abort)) {
-                            report(p.status, abort, 1, 1000 + j);
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after();
-                        issue_s(g, kst);
-                    }
-                    if (!mbar_wait(smem_u32(&bars->p_full[g]), j & 1, lim, abort)) {
-                        report(p.status, abort, 1, 2000 + j);
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    issue_o(g, vst, j > 0);
-                }
+                const int sv = (2 * j + 1) % C::STAGES, sk = (2 * j + 2) % C::STAGES;
+                // V_j has been waited for; K_{j+1} is waited for inside PV_0(j);
+                // V_{j+1} inside the last group of this step.
+                if (!(ok = wait_p(0, j))) break;
+                issue_o(0, sv, j > 0, [&] { if (more) ok = wait_load(2 * j + 2); });
                 if (!ok) break;
-                if (more) umma_commit(smem_u32(&bars->kv_empty[kst]));
-                umma_commit(smem_u32(&bars->kv_empty[vst]));
+                if (ng == 2) {
+                    if (more) issue_s(0, sk, nop);
+                    else umma_commit(smem_u32(&bars->o_done[0]));
+                    if (!(ok = wait_p(1, j))) break;
+                    issue_o(1, sv, j > 0, nop);
+                    umma_commit(smem_u32(&bars->kv_empty[sv]));
+                    if (more) {
+                        issue_s(1, sk, [&] { ok = wait_load(2 * j + 3); });
+                        umma_commit(smem_u32(&bars->kv_empty[sk]));
+                    } else {
+                        umma_commit(smem_u32(&bars->o_done[1]));
+                    }
+                } else {
+                    umma_commit(smem_u32(&bars->kv_empty[sv]));
+                    if (more) {
+                        issue_s(0, sk, [&] { ok = wait_load(2 * j + 3); });
+                        umma_commit(smem_u32(&bars->kv_empty[sk]));
+                    } else {
+                        umma_commit(smem_u32(&bars->o_done[0]));
+                    }
+                }
             }
             // drain: all issued MMAs complete before TMEM is released
-            umma_commit(smem_u32(&bars->drain));
-            mbar_wait(smem_u32(&bars->drain), 0, lim, abort);
+            umma_commit(smem_u32(&bars->drain[0]));
+            mbar_wait(smem_u32(&bars->drain[0]), 0, lim, abort);
         }
+      }
     } else {
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsSm));
         // ================================ softmax groups ===============================
-        const int g = (warp - 2) >> 2;                 // 0 or 1
+        const int g = (warp >> 2) - 1;                 // 0 or 1
         const int sub = warp & 3;                      // TMEM lane quarter of this warp
         const int row = sub * 32 + lane;               // row within the tile
         const int grow = m0 + g * kBM + row;           // query row within the chunk
@@ -286,14 +297,11 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
         const uint32_t lane_off = uint32_t(sub * 32) << 16;
         const uint32_t tS = tmem + lane_off + g * kBN;
         const uint32_t tO = tmem + lane_off + 256 + g * D;
-        const uint32_t pRow = sP + g * C::P_TILE + row * 128;
         const float sl2 = p.scale_log2;
         bool ok = active;
         if (active) {
-            if (!mbar_wait(smem_u32(&bars->q_full), 0, lim, abort)) {
-                report(p.status, abort, 2 + g, -1);
-                ok = false;
-            }
+            ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&bars->q_full), 0, lim, abort));
+            if (!ok) report(p.status, abort, 2 + g, -1);
             if (ROPE && ok && grow < sd.n_q) {
                 const int f = grow / p.rope.tpf;
                 const int rem = grow - f * p.rope.tpf;
@@ -314,95 +322,109 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
         float m_run = -INFINITY;
         float l_run = 0.0f;
         for (int j = 0; j < n_tiles && ok; ++j) {
-            if (!mbar_wait(smem_u32(&bars->s_full[g]), j & 1, lim, abort)) {
+            ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&bars->s_full[g]), j & 1, lim, abort));
+            if (!ok) {
                 report(p.status, abort, 2 + g, j);
-                ok = false;
                 break;
             }
             tc_fence_after();
-            uint32_t sr[4][32];
-#pragma unroll
-            for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, sr[c]);
-            tmem_ld_wait();
-            tc_fence_before();
-            mbar_arrive(smem_u32(&bars->s_free[g]));
-
             float s[kBN];
+            {
+                uint32_t r[4][32];
 #pragma unroll
-            for (int c = 0; c < 4; ++c)
+                for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, r[c]);
+                tmem_ld_wait();
 #pragma unroll
-                for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(sr[c][i]);
+                for (int c = 0; c < 4; ++c)
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(r[c][i]);
+            }
             if (j == n_tiles - 1) {
                 const int valid = sd.n_kv - j * kBN;
 #pragma unroll
                 for (int i = 0; i < kBN; ++i)
                     if (i >= valid) s[i] = -INFINITY;
             }
-            float mx = s[0];
+            // The exponentials of the first 64 scores are computed against the running
+            // (stale) max at the same time as the row max: they only have to be redone
+            // when the max grows by more than 2^kRescaleLog2, which after the first few
+            // tiles is rare. This keeps the max reduction off the critical path.
+            const uint64_t sl2x2 = f2_pack(sl2, sl2);
+            uint32_t pk[32];
+            uint64_t acc[4] = {0, 0, 0, 0};
+            auto exp_half = [&](int h, float mref) {
+                const uint64_t negm = f2_pack(-mref, -mref);
 #pragma unroll
-            for (int i = 1; i < kBN; ++i) mx = fmaxf(mx, s[i]);
-            const float m_new = fmaxf(m_run, mx * sl2);
+                for (int i = 0; i < 32; ++i) {
+                    const int e = h * 64 + 2 * i;
+                    float x0, x1;
+                    f2_unpack(f2_fma(f2_pack(s[e], s[e + 1]), sl2x2, negm), x0, x1);
+                    const float p0 = ex2_approx(x0);
+                    const float p1 = ex2_approx(x1);
+                    acc[i & 3] = f2_add(acc[i & 3], f2_pack(p0, p1));
+                    pk[i] = pack_bf16x2(p0, p1);
+                }
+            };
+            if (j > 0) exp_half(0, m_run);
+            // row max: 8 independent 3-input max chains
+            float mx[8];
+#pragma unroll
+            for (int a = 0; a < 8; ++a) mx[a] = fmaxf(s[a], s[a + 8]);
+#pragma unroll
+            for (int i = 16; i < kBN; i += 16)
+#pragma unroll
+                for (int a = 0; a < 8; ++a) mx[a] = max3f(mx[a], s[i + a], s[i + 8 + a]);
+            const float mrow = max3f(max3f(mx[0], mx[1], mx[2]), max3f(mx[3], mx[4], mx[5]),
+                                     fmaxf(mx[6], mx[7]));
+            const float m_new = fmaxf(m_run, mrow * sl2);
             const bool need = m_new > m_run + kRescaleLog2;
             float alpha = 1.0f;
             if (need) {
                 alpha = ex2_approx(m_run - m_new);
                 m_run = m_new;
             }
-            const float neg_m = -m_run;
-            float rs = 0.0f;
-            uint32_t pk[kBN / 2];
-#pragma unroll
-            for (int i = 0; i < kBN; i += 2) {
-                const float p0 = ex2_approx(__fmaf_rn(s[i], sl2, neg_m));
-                const float p1 = ex2_approx(__fmaf_rn(s[i + 1], sl2, neg_m));
-                rs += p0 + p1;
-                pk[i >> 1] = pack_bf16x2(p0, p1);
-            }
-            l_run = l_run * alpha + rs;
-
-            if (j > 0) {
-                // PV of the previous tile must be done: P buffer reuse and O rescale
-                if (!mbar_wait(smem_u32(&bars->o_done[g]), (j - 1) & 1, lim, abort)) {
-                    report(p.status, abort, 2 + g, 3000 + j);
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-            }
-            // P row -> shared memory, K-major 128-byte swizzle (16-byte chunk c of a
-            // 128-byte row lives at chunk position c ^ (row % 8))
-#pragma unroll
-            for (int c = 0; c < kBN / 8; ++c) {
-                const int cb = c >> 3, cc = c & 7;
-                const uint32_t addr = pRow + cb * (kBM * 128) + ((cc ^ (row & 7)) << 4);
-                asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(addr),
-                             "r"(pk[4 * c]), "r"(pk[4 * c + 1]), "r"(pk[4 * c + 2]),
-                             "r"(pk[4 * c + 3])
-                             : "memory");
-            }
-            if (j > 0 && __any_sync(0xffffffffu, need)) {
+            if (j == 0 || __any_sync(0xffffffffu, need)) {
+                if (j > 0) {
+                    // S_g(j) has landed, so PV_g(j-1) is complete: O_g is stable
 #pragma unroll 1
-                for (int c = 0; c < D / 32; ++c) {
-                    uint32_t o[32];
-                    tmem_ld32(tO + c * 32, o);
-                    tmem_ld_wait();
+                    for (int c = 0; c < D / 32; ++c) {
+                        uint32_t o[32];
+                        tmem_ld32(tO + c * 32, o);
+                        tmem_ld_wait();
 #pragma unroll
-                    for (int i = 0; i < 32; ++i)
-                        o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-                    tmem_st32(tO + c * 32, o);
+                        for (int i = 0; i < 32; i += 2) {
+                            uint64_t v = f2_mul(
+                                f2_pack(__uint_as_float(o[i]), __uint_as_float(o[i + 1])),
+                                f2_pack(alpha, alpha));
+                            float lo, hi;
+                            f2_unpack(v, lo, hi);
+                            o[i] = __float_as_uint(lo);
+                            o[i + 1] = __float_as_uint(hi);
+                        }
+                        tmem_st32(tO + c * 32, o);
+                    }
                 }
-                tmem_st_wait();
+                acc[0] = acc[1] = acc[2] = acc[3] = 0;
+                exp_half(0, m_run);
             }
-            fence_proxy_async_smem();
+            tmem_st32(tS, pk);
+            exp_half(1, m_run);
+            tmem_st32(tS + 32, pk);
+            float a0, a1, b0, b1, c0, c1, d0, d1;
+            f2_unpack(acc[0], a0, a1);
+            f2_unpack(acc[1], b0, b1);
+            f2_unpack(acc[2], c0, c1);
+            f2_unpack(acc[3], d0, d1);
+            l_run = l_run * alpha + (((a0 + a1) + (b0 + b1)) + ((c0 + c1) + (d0 + d1)));
+            tmem_st_wait();
             tc_fence_before();
             mbar_arrive(smem_u32(&bars->p_full[g]));
         }
         // ---- epilogue: O / l -> global -------------------------------------------------
         if (ok) {
-            if (!mbar_wait(smem_u32(&bars->o_done[g]), (n_tiles - 1) & 1, lim, abort)) {
-                report(p.status, abort, 2 + g, 4000);
-                ok = false;
-            }
+            ok = __all_sync(0xffffffffu,
+                            mbar_wait(smem_u32(&bars->o_done[g]), 0, lim, abort));
+            if (!ok) report(p.status, abort, 2 + g, 4000);
         }
         if (ok) {
             tc_fence_after();
@@ -458,8 +480,14 @@ cudaError_t launch(const AttnParams<MAXS>& p, cudaStream_t st) {
     auto kern = attn_kernel<D, MAXS, ROPE>;
     static bool attr_set = false;
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             Cfg<D>::SMEM);
+        // the setmaxnreg split assumes exactly kRegsLaunch registers per thread at launch;
+        // any other allocation could leave the increase waiting, so refuse to launch
+        cudaFuncAttributes fa;
+        cudaError_t e = cudaFuncGetAttributes(&fa, kern);
+        if (e != cudaSuccess) return e;
+        if (fa.numRegs != kRegsLaunch) return cudaErrorInvalidConfiguration;
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 Cfg<D>::SMEM);
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
