@@ -73,6 +73,7 @@ struct Bars {
     uint64_t kv_empty[8];
     uint32_t tmem_base;
     int abort_flag;
+    int last_split;
 };
 
 __device__ __forceinline__ void report(DeviceStatus* st, volatile int* abort, int role, int where) {
@@ -86,6 +87,22 @@ __device__ __forceinline__ void report(DeviceStatus* st, volatile int* abort, in
             __threadfence_system();
             s->code = kTimeoutCode;
         }
+    }
+}
+
+// 32 consecutive output values of one row -> fp32 or bf16 output
+__device__ __forceinline__ void store_row32(void* out, int out_bf16, size_t off, const float (&v)[32]) {
+    if (out_bf16) {
+        uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(out) + off);
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            dst[i] = make_uint4(pack_bf16x2(v[8 * i + 0], v[8 * i + 1]), pack_bf16x2(v[8 * i + 2], v[8 * i + 3]),
+                                pack_bf16x2(v[8 * i + 4], v[8 * i + 5]), pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
+    } else {
+        float4* dst = reinterpret_cast<float4*>(static_cast<float*>(out) + off);
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+            dst[i] = make_float4(v[4 * i + 0], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
     }
 }
 
@@ -106,12 +123,20 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
     int si = 0;
     while (si + 1 < p.n_streams && item >= p.s[si + 1].item_begin) ++si;
     const AttnStreamDesc& sd = p.s[si];
+    // items of a stream: ((head * n_split + split) * n_qpairs + pair), so CTAs launched
+    // together share one head's K/V range
     const int local = item - sd.item_begin;
-    const int head = local / sd.n_qpairs;
-    const int m0 = (local - head * sd.n_qpairs) * (2 * kBM);
+    const int hs = local / sd.n_qpairs;
+    const int pair = local - hs * sd.n_qpairs;
+    const int head = hs / p.n_split;
+    const int split = hs - head * p.n_split;
+    const int group = sd.group_begin + head * sd.n_qpairs + pair;
+    const int m0 = pair * (2 * kBM);
     const bool active1 = (m0 + kBM) < sd.n_q;
     const int ng = active1 ? 2 : 1;
-    const int n_tiles = (sd.n_kv + kBN - 1) / kBN;
+    const int tiles_total = (sd.n_kv + kBN - 1) / kBN;
+    const int t0 = split * tiles_total / p.n_split;          // this split's KV tiles
+    const int n_tiles = (split + 1) * tiles_total / p.n_split - t0;
     const int n_loads = 2 * n_tiles;
 
     const int warp = threadIdx.x >> 5;
@@ -169,7 +194,7 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                     break;
                 }
                 const CUtensorMap* map = (L & 1) ? &sd.v_map : &sd.k_map;
-                const int row = (L >> 1) * kBN;
+                const int row = (t0 + (L >> 1)) * kBN;
                 const uint32_t fb = smem_u32(&bars->kv_full[stage]);
                 mbar_arrive_expect_tx(fb, C::KV_TILE);
                 const uint32_t dst = sKV + stage * C::KV_TILE;
@@ -339,8 +364,8 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
 #pragma unroll
                     for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(r[c][i]);
             }
-            if (j == n_tiles - 1) {
-                const int valid = sd.n_kv - j * kBN;
+            if (t0 + j == tiles_total - 1) {
+                const int valid = sd.n_kv - (t0 + j) * kBN;
 #pragma unroll
                 for (int i = 0; i < kBN; ++i)
                     if (i >= valid) s[i] = -INFINITY;
@@ -420,49 +445,92 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             tc_fence_before();
             mbar_arrive(smem_u32(&bars->p_full[g]));
         }
-        // ---- epilogue: O / l -> global -------------------------------------------------
+        // ---- epilogue ------------------------------------------------------------------
         if (ok) {
             ok = __all_sync(0xffffffffu,
                             mbar_wait(smem_u32(&bars->o_done[g]), 0, lim, abort));
             if (!ok) report(p.status, abort, 2 + g, 4000);
         }
-        if (ok) {
+        const bool store = ok && grow < sd.n_q;
+        const size_t obase = (size_t(grow) * p.heads + head) * D;
+        if (ok && p.n_split == 1) {
+            // O / l -> out
             tc_fence_after();
             const float inv_l = 1.0f / l_run;
-            const bool store = grow < sd.n_q;
-            const size_t obase = (size_t(grow) * p.heads + head) * D;
 #pragma unroll 1
             for (int c = 0; c < D / 32; ++c) {
                 uint32_t o[32];
                 tmem_ld32(tO + c * 32, o);
                 tmem_ld_wait();
                 if (store) {
-                    if (p.out_bf16) {
-                        uint4* dst = reinterpret_cast<uint4*>(
-                            static_cast<uint16_t*>(sd.out) + obase + c * 32);
+                    float v[32];
 #pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            uint4 w;
-                            w.x = pack_bf16x2(__uint_as_float(o[8 * i + 0]) * inv_l,
-                                              __uint_as_float(o[8 * i + 1]) * inv_l);
-                            w.y = pack_bf16x2(__uint_as_float(o[8 * i + 2]) * inv_l,
-                                              __uint_as_float(o[8 * i + 3]) * inv_l);
-                            w.z = pack_bf16x2(__uint_as_float(o[8 * i + 4]) * inv_l,
-                                              __uint_as_float(o[8 * i + 5]) * inv_l);
-                            w.w = pack_bf16x2(__uint_as_float(o[8 * i + 6]) * inv_l,
-                                              __uint_as_float(o[8 * i + 7]) * inv_l);
-                            dst[i] = w;
+                    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(o[i]) * inv_l;
+                    store_row32(sd.out, p.out_bf16, obase + c * 32, v);
+                }
+            }
+        } else if (ok) {
+            // unnormalised partial of this split -> scratch
+            tc_fence_after();
+            const size_t prow = (size_t(group) * p.n_split + split) * 2 * kBM + g * kBM + row;
+            float4* po = reinterpret_cast<float4*>(p.part_o + prow * D);
+#pragma unroll 1
+            for (int c = 0; c < D / 32; ++c) {
+                uint32_t o[32];
+                tmem_ld32(tO + c * 32, o);
+                tmem_ld_wait();
+#pragma unroll
+                for (int i = 0; i < 8; ++i)
+                    po[c * 8 + i] = make_float4(__uint_as_float(o[4 * i]), __uint_as_float(o[4 * i + 1]),
+                                                __uint_as_float(o[4 * i + 2]), __uint_as_float(o[4 * i + 3]));
+            }
+            p.part_ml[prow] = make_float2(m_run, l_run);
+            __threadfence();
+        }
+        if (p.n_split > 1) {
+            // the last split of this query group to finish merges all partials
+            named_bar_sync(1, 256);
+            if (threadIdx.x == 128) {
+                const int old = atomicAdd(p.counters + group, 1);
+                const int last = (old == p.n_split - 1);
+                if (last) p.counters[group] = 0;   // every split has counted: reset for reuse
+                bars->last_split = last;
+            }
+            named_bar_sync(1, 256);
+            if (bars->last_split && store) {
+                __threadfence();
+                const size_t prow0 = size_t(group) * p.n_split * 2 * kBM + g * kBM + row;
+                float mref = -INFINITY;
+                for (int r = 0; r < p.n_split; ++r)
+                    mref = fmaxf(mref, __ldcg(&p.part_ml[prow0 + size_t(r) * 2 * kBM]).x);
+                float lsum = 0.0f;
+                for (int r = 0; r < p.n_split; ++r) {
+                    const float2 ml = __ldcg(&p.part_ml[prow0 + size_t(r) * 2 * kBM]);
+                    lsum += ex2_approx(ml.x - mref) * ml.y;
+                }
+                const float inv_l = 1.0f / lsum;
+#pragma unroll 1
+                for (int c = 0; c < D / 32; ++c) {
+                    float v[32];
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] = 0.0f;
+                    for (int r = 0; r < p.n_split; ++r) {
+                        const float w = ex2_approx(
+                            __ldcg(&p.part_ml[prow0 + size_t(r) * 2 * kBM]).x - mref);
+                        const float4* src = reinterpret_cast<const float4*>(
+                            p.part_o + (prow0 + size_t(r) * 2 * kBM) * D + c * 32);
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const float4 x = __ldcg(src + i);
+                            v[4 * i] += w * x.x;
+                            v[4 * i + 1] += w * x.y;
+                            v[4 * i + 2] += w * x.z;
+                            v[4 * i + 3] += w * x.w;
                         }
-                    } else {
-                        float4* dst = reinterpret_cast<float4*>(
-                            static_cast<float*>(sd.out) + obase + c * 32);
-#pragma unroll
-                        for (int i = 0; i < 8; ++i)
-                            dst[i] = make_float4(__uint_as_float(o[4 * i + 0]) * inv_l,
-                                                 __uint_as_float(o[4 * i + 1]) * inv_l,
-                                                 __uint_as_float(o[4 * i + 2]) * inv_l,
-                                                 __uint_as_float(o[4 * i + 3]) * inv_l);
                     }
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] *= inv_l;
+                    store_row32(sd.out, p.out_bf16, obase + c * 32, v);
                 }
             }
         }

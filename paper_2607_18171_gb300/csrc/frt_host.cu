@@ -104,6 +104,13 @@ struct frt_stream {
     cudaEvent_t ev = nullptr;   // cross-stream ordering for batched launches
     cudaEvent_t attn_start = nullptr;  // caller-owned instrumentation events
     cudaEvent_t attn_stop = nullptr;
+    // split-KV scratch: partial O / (max, sum) per (query group, split), one counter per
+    // query group (zero between launches)
+    float* part_o = nullptr;
+    float2* part_ml = nullptr;
+    int* counters = nullptr;
+    long long part_groups = 0;   // capacity: query groups
+    int part_splits = 1;         // capacity: splits per group
 };
 
 namespace {
@@ -144,6 +151,53 @@ void fill_rope(const frt_stream_t* s, long long c, RopeArgs& a) {
     }
 }
 
+// Split-KV factor for `groups` query groups of `tiles` KV tiles each: minimise the
+// makespan ceil(groups * s / SMs) / s, with a 2 % cost per extra split (the partial
+// round trip and merge); each split keeps at least two KV tiles.
+int choose_split(long long groups, int tiles, int max_split) {
+    const long long sms = num_sms();
+    int best = 1;
+    double best_t = double((groups + sms - 1) / sms);
+    for (int sp = 2; sp <= max_split && sp <= kMaxSplit; ++sp) {
+        if (tiles < 2 * sp) break;
+        const double t = double((groups * sp + sms - 1) / sms) / sp * (1.0 + 0.02 * (sp - 1));
+        if (t < best_t - 1e-9) {
+            best_t = t;
+            best = sp;
+        }
+    }
+    return best;
+}
+
+// Make sure s owns split-KV scratch for `groups` query groups x `splits` splits
+// (allocates, synchronously, only when it must grow).
+frt_status ensure_scratch(frt_stream_t* s, long long groups, int splits) {
+    if (splits <= 1 || (groups <= s->part_groups && splits <= s->part_splits)) return FRT_OK;
+    cudaError_t e;
+    if (s->part_o && (e = cudaStreamSynchronize(s->cs)) != cudaSuccess)
+        return cuda_fail(e, "sync before scratch growth");
+    const long long g = std::max(groups, s->part_groups);
+    const int sp = std::max(splits, s->part_splits);
+    if (s->part_o) cudaFree(s->part_o);
+    if (s->part_ml) cudaFree(s->part_ml);
+    if (s->counters) cudaFree(s->counters);
+    s->part_o = nullptr;
+    s->part_ml = nullptr;
+    s->counters = nullptr;
+    s->part_groups = 0;
+    s->part_splits = 1;
+    const size_t rows = size_t(g) * sp * 2 * 128;
+    if ((e = cudaMalloc(&s->part_o, rows * s->head_dim * sizeof(float))) != cudaSuccess ||
+        (e = cudaMalloc(&s->part_ml, rows * sizeof(float2))) != cudaSuccess ||
+        (e = cudaMalloc(&s->counters, size_t(g) * sizeof(int))) != cudaSuccess ||
+        (e = cudaMemset(s->counters, 0, size_t(g) * sizeof(int))) != cudaSuccess ||
+        (e = cudaDeviceSynchronize()) != cudaSuccess)
+        return cuda_fail(e, "split-KV scratch allocation");
+    s->part_groups = g;
+    s->part_splits = sp;
+    return FRT_OK;
+}
+
 int log2_exact(int x) {
     int l = 0;
     while ((1 << l) < x) ++l;
@@ -165,9 +219,15 @@ frt_status attention_single(frt_stream_t* s, const void* q, void* out, bool rope
     d.n_kv = int(n_kv);
     d.n_qpairs = (s->n_q + 255) / 256;
     d.item_begin = 0;
+    d.group_begin = 0;
+    const long long groups = (long long)d.n_qpairs * s->heads;
+    p.n_split = choose_split(groups, int((n_kv + 127) / 128), s->part_splits);
+    p.part_o = s->part_o;
+    p.part_ml = s->part_ml;
+    p.counters = s->counters;
     p.n_streams = 1;
     p.heads = s->heads;
-    p.total_items = d.n_qpairs * s->heads;
+    p.total_items = int(groups * p.n_split);
     p.out_bf16 = s->cfg.out_dtype == FRT_OUT_BF16;
     p.scale_log2 = float(double(s->scale) * 1.4426950408889634);
     p.wait_limit_ns = s->wait_limit_ns;
@@ -217,6 +277,14 @@ void free_device(frt_stream_t* s) {
     if (s->status_host) cudaFreeHost(s->status_host);
     if (s->ev) cudaEventDestroy(s->ev);
     s->ev = nullptr;
+    if (s->part_o) cudaFree(s->part_o);
+    if (s->part_ml) cudaFree(s->part_ml);
+    if (s->counters) cudaFree(s->counters);
+    s->part_o = nullptr;
+    s->part_ml = nullptr;
+    s->counters = nullptr;
+    s->part_groups = 0;
+    s->part_splits = 1;
     s->cache_k = s->cache_v = nullptr;
     s->d_hw = nullptr;
     s->stage = nullptr;
@@ -369,6 +437,16 @@ frt_status frt_stream_configure(frt_stream_t* s, const frt_config* cfg) {
                         cudaMemcpyHostToDevice)) != cudaSuccess)
         return cuda_fail(e, "rope table upload");
     s->hw_entries = int(hw.size());
+    {
+        // split-KV scratch for the steady-state (full window) launch of this stream
+        const long long groups = (long long)((s->n_q + 255) / 256) * s->heads;
+        const int tiles = int(((long long)s->window * s->n_q + 127) / 128);
+        frt_status st = ensure_scratch(s, groups, choose_split(groups, tiles, kMaxSplit));
+        if (st != FRT_OK) {
+            free_device(s);
+            return st;
+        }
+    }
     // zero cache: rows past the valid prefix are never read by value, but keep them finite
     if ((e = cudaMemset(s->cache_k, 0, cache_bytes)) != cudaSuccess ||
         (e = cudaMemset(s->cache_v, 0, cache_bytes)) != cudaSuccess)
@@ -505,7 +583,22 @@ frt_status frt_chunk_attention_batched(frt_stream_t* const* streams, int n, cons
     auto* p = new (std::nothrow) AttnParams<kMaxBatchStreams>();
     if (!p) return fail(FRT_ERR_OOM, "host allocation failed");
     std::memset(p, 0, sizeof(*p));
-    int items = 0;
+    long long groups_total = 0;
+    int min_tiles = 1 << 30;
+    for (int i = 0; i < n; ++i) {
+        groups_total += (long long)((streams[i]->n_q + 255) / 256) * streams[i]->heads;
+        min_tiles = std::min(min_tiles, int((n_kv(i) + 127) / 128));
+    }
+    const int n_split = choose_split(groups_total, min_tiles, kMaxSplit);
+    if ((st = ensure_scratch(s0, groups_total, n_split)) != FRT_OK) {
+        delete p;
+        return st;
+    }
+    p->n_split = n_split;
+    p->part_o = s0->part_o;
+    p->part_ml = s0->part_ml;
+    p->counters = s0->counters;
+    int items = 0, groups = 0;
     for (int oi = 0; oi < n; ++oi) {
         const int i = order[oi];
         frt_stream_t* s = streams[i];
@@ -522,7 +615,9 @@ frt_status frt_chunk_attention_batched(frt_stream_t* const* streams, int n, cons
         d.n_kv = int(nkv);
         d.n_qpairs = (s->n_q + 255) / 256;
         d.item_begin = items;
-        items += d.n_qpairs * s->heads;
+        d.group_begin = groups;
+        items += d.n_qpairs * s->heads * n_split;
+        groups += d.n_qpairs * s->heads;
     }
     p->n_streams = n;
     p->heads = s0->heads;

@@ -10,6 +10,8 @@ namespace frt {
 constexpr int kMaxTEntries = 256;
 // Largest number of streams in one batched attention launch.
 constexpr int kMaxBatchStreams = 32;
+// Largest split-KV factor (KV ranges per query group).
+constexpr int kMaxSplit = 4;
 
 // Device status block (host-mapped pinned memory): the first device error wins.
 struct DeviceStatus {
@@ -73,8 +75,9 @@ struct AttnStreamDesc {
     void* out;           // [Nq, H, D] fp32 or bf16
     int n_q;
     int n_kv;
-    int n_qpairs;        // ceil(Nq / 256): work items per head
+    int n_qpairs;        // ceil(Nq / 256): query groups per head
     int item_begin;      // first work item of this stream
+    int group_begin;     // first query group (head, 256 rows) of this stream
 };
 
 template <int MAXS>
@@ -85,6 +88,13 @@ struct AttnParams {
     int total_items;
     int out_bf16;
     float scale_log2;            // sm_scale * log2(e)
+    // Split-KV: each query group's KV tiles are cut into n_split contiguous ranges
+    // processed by separate CTAs; each writes an unnormalised partial (O, running max,
+    // row sum) and the last to finish merges them. n_split == 1 uses none of these.
+    int n_split;
+    float* part_o;               // [groups * n_split][2][128][D] fp32
+    float2* part_ml;             // [groups * n_split][2][128] (max in log2 units, sum)
+    int* counters;               // [groups], zero between launches
     unsigned long long wait_limit_ns;
     DeviceStatus* status;
     RopeArgs rope;               // RoPE-Q prologue (single-stream fused path only)

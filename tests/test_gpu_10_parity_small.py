@@ -149,7 +149,11 @@ def test_batched_ragged_streams_match_single_launches_and_oracle(frt):
         outs_s.append(o)
     torch.cuda.synchronize()
     for s, fill in enumerate(fills):
-        assert torch.equal(outs_b[s], outs_s[s]), s
+        # the two launches may pick different split-KV factors (the batched one sees
+        # more query groups); each split rounds P to bf16 against its own running max,
+        # so the two agree to the bf16 rounding of P, not bit for bit
+        max_abs, rel = U.compare(outs_b[s].cpu().numpy(), outs_s[s].cpu().numpy())
+        assert max_abs <= 5e-3 and rel <= 2e-3, (s, max_abs, rel)
         ref = U.oracle_full_stream(base, s, fill)[fill - 1][0]
         U.assert_close(outs_b[s].cpu().numpy(), ref, f"stream {s}")
     for st in streams:
