@@ -135,6 +135,35 @@ frt_status frt_chunk_step_host(frt_stream_t* s, const void* q_host,
 frt_status frt_chunk_attention_batched(frt_stream_t* const* streams, int n,
                                        const void* const* q, void* const* out);
 
+/* Operation 3 for callers that cannot allocate device memory (no counterpart in
+ * the paper). Some callers may not call cudaMalloc: code under a memory planner or
+ * arena that owns every device byte, real-time loops where an allocation (which can
+ * synchronise the device) is not allowed, integrations whose only device memory is
+ * what they pass in. This call allocates nothing: no stream handle, no cudaMalloc,
+ * cudaFree or allocating library routine. It computes the same attention as
+ * frt_chunk_attention, out[i,h,:] = sum_j softmax_j(scale <q[i,h], k[j,h]>) v[j,h,:]
+ * over all n_kv rows of caller-owned buffers:
+ *   q    device [n_q, heads, head_dim] bf16 (already rotated);
+ *   k, v device [n_kv, heads, head_dim] bf16 (e.g. the valid prefix of a cache);
+ *   out  device [n_q, heads, head_dim], fp32 or bf16 (out_dtype);
+ *   sm_scale <= 0 selects 1/sqrt(head_dim);
+ *   status optional device pointer to 4 ints, zeroed by the caller, where a device
+ *        bounded-wait timeout records FRT_ERR_TIMEOUT (NULL: not recorded);
+ *   cuda_stream the cudaStream_t the work is enqueued on (NULL = legacy stream).
+ * All pointers 16-byte aligned; head_dim 64 or 128. The kernel's split-KV scratch
+ * lives in one static device array of this library (8 MiB of partials, 4096 merge
+ * counters) that every GPU loading the library holds until exit; splits are limited
+ * to what it holds, and heads * ceil(n_q / 256) > 4096 is rejected with
+ * FRT_ERR_UNSUPPORTED. The first call on a device looks up the array's device
+ * address; make that first call before any stream capture. All calls share the
+ * array and each clears its merge counters on the stream first: calls that overlap
+ * on the GPU (other streams, other threads) race and must not be issued.
+ * frt_last_error() describes an error this call returns. */
+frt_status frt_chunk_attention_noalloc(const void* q, const void* k, const void* v,
+                                       void* out, int n_q, int n_kv, int heads,
+                                       int head_dim, double sm_scale, int out_dtype,
+                                       void* status, void* cuda_stream);
+
 /* Wait for the stream's work and return its device status (FRT_OK or the
  * first device error, e.g. FRT_ERR_TIMEOUT). */
 frt_status frt_stream_sync(frt_stream_t* s);

@@ -705,6 +705,8 @@ frt_status frt_stream_cache(const frt_stream_t* s, const void** k_cache, const v
 
 }  // extern "C"
 
+void frt::set_last_error(const char* msg) { g_last_error = msg; }
+
 // Device pointer of a stream's status block (used by the self-test entry points).
 extern "C" void* frt_internal_status_dev(frt_stream_t* s) {
     return (s && s->configured) ? static_cast<void*>(s->status_dev) : nullptr;

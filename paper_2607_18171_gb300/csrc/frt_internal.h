@@ -129,5 +129,7 @@ cudaError_t launch_attention_single(const AttnParams<1>& p, int head_dim, bool r
 cudaError_t launch_attention_batched(const AttnParams<kMaxBatchStreams>& p, int head_dim,
                                      cudaStream_t st);
 int num_sms();
+// Set the thread-local message that frt_last_error() returns.
+void set_last_error(const char* msg);
 
 }  // namespace frt
