@@ -189,6 +189,7 @@ def run_gpu(args, wl, world, rank, local):
     st.sync()
     n = args.steps
     ev_a = timing_events(n, stream)
+    ev_k = timing_events(n, stream)
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     if world > 1:
         torch.distributed.barrier()
@@ -197,15 +198,19 @@ def run_gpu(args, wl, world, rank, local):
         t0.record(stream)
         for i in range(n):
             st.set_attention_events(*ev_a[i])
+            st.set_append_events(*ev_k[i])
             step(args.warmup + i)
         t1.record(stream)
         torch.cuda.synchronize()
     st.set_attention_events(None, None)
+    st.set_append_events(None, None)
     st.sync()
     if world > 1:
         torch.distributed.barrier()
     elapsed_ms = t0.elapsed_time(t1)
     attn_ms = [a.elapsed_time(b) for a, b in ev_a]
+    app_ms = statistics.mean(a.elapsed_time(b) for a, b in ev_k)
+    app_bytes = 2 * 2 * wl.n_q * wl.heads * wl.head_dim * 2   # read + write of K and V
     wall_ms = max_over_ranks(elapsed_ms, world, dev)
     total_flops = flops * n * world
     value = total_flops / (wall_ms * 1e-3) / 1e12
@@ -253,6 +258,12 @@ def run_gpu(args, wl, world, rank, local):
                      "traffic": traffic, "kernel": "attn_kernel<128,1,true>",
                      "peak_kind": f"{peak_kind} bf16 dense burst",
                      "launch_ms": round(attn_mean, 4)},
+        "append": {"bound": "hbm", "achieved": round(app_bytes / (app_ms * 1e-3) / 1e9, 1),
+                   "peak": peak_gbs, "unit": "GB/s",
+                   "frac": round(app_bytes / (app_ms * 1e-3) / 1e9 / peak_gbs, 4),
+                   "frac_of_8tbs": round(app_bytes / (app_ms * 1e-3) / 8e12, 4),
+                   "kernel": "kv_append_kernel (RoPE-K fused)", "launch_ms": round(app_ms, 5),
+                   "bytes_per_launch": app_bytes},
         "clocks": clk.summary(),
         "e2e": {"value": round(e2e_value, 2), "unit": UNIT,
                 "h2d_bytes_per_step": 3 * wl.n_q * wl.heads * wl.head_dim * 2,

@@ -187,6 +187,10 @@ frt_status frt_stream_cache(const frt_stream_t* s, const void** k_cache,
 frt_status frt_stream_set_attention_events(frt_stream_t* s, void* start_event,
                                            void* stop_event);
 
+/* Instrumentation: the same for every KV append kernel launch of s
+ * (frt_kv_append_evict and the append inside frt_chunk_step). */
+frt_status frt_stream_set_append_events(frt_stream_t* s, void* start_event, void* stop_event);
+
 /* Index of the next chunk to be appended (chunks appended so far). */
 long long frt_stream_chunk_counter(const frt_stream_t* s);
 

@@ -104,6 +104,8 @@ struct frt_stream {
     cudaEvent_t ev = nullptr;   // cross-stream ordering for batched launches
     cudaEvent_t attn_start = nullptr;  // caller-owned instrumentation events
     cudaEvent_t attn_stop = nullptr;
+    cudaEvent_t app_start = nullptr;
+    cudaEvent_t app_stop = nullptr;
     // split-KV scratch: partial O / (max, sum) per (query group, split), one counter per
     // query group (zero between launches)
     float* part_o = nullptr;
@@ -258,7 +260,10 @@ frt_status append_impl(frt_stream_t* s, const void* k, const void* v, bool rope_
     p.vec_per_head_log2 = log2_exact(s->head_dim / 8);
     p.rope = rope_k ? 1 : 0;
     if (rope_k) fill_rope(s, s->counter, p.ra);
-    cudaError_t e = launch_kv_append(p, s->cs);
+    cudaError_t e = cudaSuccess;
+    if (s->app_start) e = cudaEventRecord(s->app_start, s->cs);
+    if (e == cudaSuccess) e = launch_kv_append(p, s->cs);
+    if (e == cudaSuccess && s->app_stop) e = cudaEventRecord(s->app_stop, s->cs);
     if (e != cudaSuccess) return cuda_fail(e, "append launch");
     s->counter += 1;
     s->phase = kAppended;
@@ -690,6 +695,15 @@ frt_status frt_stream_set_attention_events(frt_stream_t* s, void* start_event,
         return fail(FRT_ERR_INVALID_ARG, "give both events or neither");
     s->attn_start = static_cast<cudaEvent_t>(start_event);
     s->attn_stop = static_cast<cudaEvent_t>(stop_event);
+    return FRT_OK;
+}
+
+frt_status frt_stream_set_append_events(frt_stream_t* s, void* start_event, void* stop_event) {
+    if (!s) return fail(FRT_ERR_INVALID_ARG, "NULL stream handle");
+    if ((start_event == nullptr) != (stop_event == nullptr))
+        return fail(FRT_ERR_INVALID_ARG, "give both events or neither");
+    s->app_start = static_cast<cudaEvent_t>(start_event);
+    s->app_stop = static_cast<cudaEvent_t>(stop_event);
     return FRT_OK;
 }
 

@@ -64,6 +64,8 @@ def lib() -> ctypes.CDLL:
         "frt_stream_chunk_counter": (LL, [P]),
         "frt_stream_cache": (I, [P, ctypes.POINTER(P), ctypes.POINTER(P), ctypes.POINTER(LL)]),
         "frt_stream_set_attention_events": (I, [P, P, P]),
+        "frt_stream_set_append_events": (I, [P, P, P]),
+        "frt_chunk_attention_noalloc": (I, [P, P, P, P, I, I, I, I, D, I, P, P]),
         "frt_window_index": (I, [LL, I, ctypes.POINTER(I), ctypes.POINTER(LL),
                                  ctypes.POINTER(I)]),
         "frt_status_string": (ctypes.c_char_p, [I]),
@@ -76,7 +78,6 @@ def lib() -> ctypes.CDLL:
         fn = getattr(L, name)
         fn.restype = res
         fn.argtypes = args
-    _ = D
     _lib = L
     return L
 
@@ -208,6 +209,13 @@ class Stream:
                              stop: torch.cuda.Event | None) -> None:
         """Record these events around every attention kernel launch of this stream."""
         _check(lib().frt_stream_set_attention_events(
+            self._h, None if start is None else ctypes.c_void_p(start.cuda_event),
+            None if stop is None else ctypes.c_void_p(stop.cuda_event)))
+
+    def set_append_events(self, start: torch.cuda.Event | None,
+                          stop: torch.cuda.Event | None) -> None:
+        """Record these events around every KV append kernel launch of this stream."""
+        _check(lib().frt_stream_set_append_events(
             self._h, None if start is None else ctypes.c_void_p(start.cuda_event),
             None if stop is None else ctypes.c_void_p(stop.cuda_event)))
 
