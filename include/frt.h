@@ -63,7 +63,7 @@ typedef struct frt_config {
 } frt_config;
 
 /* Create a stream handle.
- *   heads >= 1; head_dim in {64, 128}; tokens_per_frame >= 1;
+ *   heads >= 1; head_dim in {64, 128}; heads * head_dim <= 12800; tokens_per_frame >= 1;
  *   frames_per_chunk >= 1; window_chunks >= 1 (the window counts the current chunk).
  * Nq = frames_per_chunk * tokens_per_frame must be <= 2^20 and
  * window_chunks * Nq <= 2^24. Allocates no device memory.
@@ -118,8 +118,12 @@ frt_status frt_chunk_step(frt_stream_t* s, const void* q, const void* k,
 
 /* frt_chunk_step with HOST buffers: copies q, k, v host -> device into
  * stream-owned staging buffers, runs the fused step, copies out device ->
- * host, all enqueued on the stream. Host buffers must stay valid until
- * frt_stream_sync returns (pinned memory makes the copies asynchronous). */
+ * host. Consecutive calls are pipelined: two staging sets alternate, the copies
+ * in run on an internal copy stream while the previous call's kernels run, and
+ * the copy out on another while the next call computes (events keep every set's
+ * reuse ordered). Host buffers must stay valid, and out_host unread, until
+ * frt_stream_sync returns (pinned memory makes the copies asynchronous). The
+ * staging (2 x (3 inputs + output)) is allocated on the first call. */
 frt_status frt_chunk_step_host(frt_stream_t* s, const void* q_host,
                                const void* k_host, const void* v_host,
                                void* out_host, int* slot_out,

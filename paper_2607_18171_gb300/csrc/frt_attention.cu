@@ -204,9 +204,9 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             // drain: every issued load must have landed before the CTA may exit
             const int first = (L - C::STAGES) > 0 ? (L - C::STAGES) : 0;
             for (int Ld = first; Ld < L; ++Ld)
-                mbar_wait(smem_u32(&bars->kv_full[Ld % C::STAGES]), (Ld / C::STAGES) & 1,
-                          lim, abort);
-            mbar_wait(qbar, 0, lim, abort);
+                mbar_wait_drain(smem_u32(&bars->kv_full[Ld % C::STAGES]), (Ld / C::STAGES) & 1,
+                                lim);
+            mbar_wait_drain(qbar, 0, lim);
         }
       } else if (warp == 1) {
         // ============ MMA issuer: one thread, tiles alternate on the tensor pipe ============
@@ -308,7 +308,7 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             }
             // drain: all issued MMAs complete before TMEM is released
             umma_commit(smem_u32(&bars->drain[0]));
-            mbar_wait(smem_u32(&bars->drain[0]), 0, lim, abort);
+            mbar_wait_drain(smem_u32(&bars->drain[0]), 0, lim);
         }
       }
     } else {
@@ -338,7 +338,7 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                     const int cb = c >> 3, cc = c & 7;
                     uint4* ptr = reinterpret_cast<uint4*>(qrow + cb * (kBM * 128) +
                                                           ((cc ^ (row & 7)) << 4));
-                    *ptr = rope_rotate8(*ptr, c * 8, f, rr, col, p.rope);
+                    *ptr = rope_rotate8(*ptr, c * 8, f, rr, col, p.rope, p.rope.t_tab);
                 }
                 fence_proxy_async_smem();
             }

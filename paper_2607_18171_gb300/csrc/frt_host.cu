@@ -98,8 +98,14 @@ struct frt_stream {
     const void* last_q = nullptr;
     const void* last_k = nullptr;
     const void* last_v = nullptr;
-    void* stage = nullptr;      // host-API staging: q, k, v (bf16) and out
+    void* stage = nullptr;      // host-API staging: two sets of q, k, v (bf16) and out
     size_t stage_bytes = 0;
+    int stage_turn = 0;         // staging set of the next host-buffer step
+    cudaStream_t cp_in = nullptr;   // host-to-device copies of host-buffer steps
+    cudaStream_t cp_out = nullptr;  // device-to-host copies of host-buffer steps
+    cudaEvent_t ev_in[2] = {nullptr, nullptr};    // inputs of set b landed
+    cudaEvent_t ev_done[2] = {nullptr, nullptr};  // kernels reading set b finished
+    cudaEvent_t ev_out[2] = {nullptr, nullptr};   // output of set b copied out
     unsigned long long wait_limit_ns = kDefaultWaitLimitNs;
     cudaEvent_t ev = nullptr;   // cross-stream ordering for batched launches
     cudaEvent_t attn_start = nullptr;  // caller-owned instrumentation events
@@ -259,6 +265,7 @@ frt_status append_impl(frt_stream_t* s, const void* k, const void* v, bool rope_
     p.vec_per_tok = s->heads * s->head_dim / 8;
     p.vec_per_head_log2 = log2_exact(s->head_dim / 8);
     p.rope = rope_k ? 1 : 0;
+    p.status = s->status_dev;
     if (rope_k) fill_rope(s, s->counter, p.ra);
     cudaError_t e = cudaSuccess;
     if (s->app_start) e = cudaEventRecord(s->app_start, s->cs);
@@ -282,6 +289,17 @@ void free_device(frt_stream_t* s) {
     if (s->status_host) cudaFreeHost(s->status_host);
     if (s->ev) cudaEventDestroy(s->ev);
     s->ev = nullptr;
+    if (s->cp_in) cudaStreamSynchronize(s->cp_in);
+    if (s->cp_out) cudaStreamSynchronize(s->cp_out);
+    for (int b = 0; b < 2; ++b) {
+        if (s->ev_in[b]) cudaEventDestroy(s->ev_in[b]);
+        if (s->ev_done[b]) cudaEventDestroy(s->ev_done[b]);
+        if (s->ev_out[b]) cudaEventDestroy(s->ev_out[b]);
+        s->ev_in[b] = s->ev_done[b] = s->ev_out[b] = nullptr;
+    }
+    if (s->cp_in) cudaStreamDestroy(s->cp_in);
+    if (s->cp_out) cudaStreamDestroy(s->cp_out);
+    s->cp_in = s->cp_out = nullptr;
     if (s->part_o) cudaFree(s->part_o);
     if (s->part_ml) cudaFree(s->part_ml);
     if (s->counters) cudaFree(s->counters);
@@ -337,7 +355,14 @@ frt_stream_t* frt_stream_create(int heads, int head_dim, int tokens_per_frame,
         return nullptr;
     }
     const long long n_q = (long long)frames_per_chunk * tokens_per_frame;
-    if (n_q > (1 << 20) || n_q * window_chunks > (1 << 24) || heads > 1024) {
+    if ((long long)heads * head_dim > 12800) {
+        // the staged append/RoPE kernel keeps 4 stages of two token rows in 200 KB of
+        // shared memory: a token row (heads * head_dim bf16) may be at most 25 KB
+        fail(FRT_ERR_UNSUPPORTED, "heads * head_dim = %lld exceeds 12800",
+             (long long)heads * head_dim);
+        return nullptr;
+    }
+    if (n_q > (1 << 20) || n_q * window_chunks > (1 << 24)) {
         fail(FRT_ERR_UNSUPPORTED, "chunk or window too large (Nq=%lld, W=%d)", n_q, window_chunks);
         return nullptr;
     }
@@ -477,6 +502,7 @@ frt_status frt_rope3d_qk(frt_stream_t* s, void* q, void* k) {
     p.n_tok = s->n_q;
     p.vec_per_tok = s->heads * s->head_dim / 8;
     p.vec_per_head_log2 = log2_exact(s->head_dim / 8);
+    p.status = s->status_dev;
     fill_rope(s, s->counter, p.ra);
     cudaError_t e = launch_rope_qk(p, s->cs);
     if (e != cudaSuccess) return cuda_fail(e, "rope launch");
@@ -528,33 +554,59 @@ frt_status frt_chunk_step_host(frt_stream_t* s, const void* q_host, const void* 
     if (st != FRT_OK) return st;
     if (!q_host || !k_host || !v_host || !out_host)
         return fail(FRT_ERR_INVALID_ARG, "NULL host buffer");
+    if (s->phase == kRoped) return fail(FRT_ERR_STATE, "a separate rope is pending");
+    // Pipelined: two staging sets alternate; the host-to-device copies of this call run
+    // on a copy stream while the previous call's kernels still run, the device-to-host
+    // copy on a third stream while the next call computes. Events order each set's
+    // reuse: copy-in(n) after compute(n-2), compute(n) after copy-in(n) and after
+    // copy-out(n-2), copy-out(n) after compute(n).
     const size_t in_bytes = s->chunk_elems * 2;
     const size_t out_bytes = s->chunk_elems * (s->cfg.out_dtype == FRT_OUT_BF16 ? 2 : 4);
-    const size_t need = 3 * in_bytes + out_bytes;
+    const size_t per_set = 3 * in_bytes + out_bytes;
     cudaError_t e;
-    if (s->stage_bytes < need) {
+    if (!s->cp_in) {
+        if ((e = cudaStreamCreateWithFlags(&s->cp_in, cudaStreamNonBlocking)) != cudaSuccess ||
+            (e = cudaStreamCreateWithFlags(&s->cp_out, cudaStreamNonBlocking)) != cudaSuccess)
+            return cuda_fail(e, "copy stream creation");
+        for (int b = 0; b < 2; ++b)
+            if ((e = cudaEventCreateWithFlags(&s->ev_in[b], cudaEventDisableTiming)) != cudaSuccess ||
+                (e = cudaEventCreateWithFlags(&s->ev_done[b], cudaEventDisableTiming)) != cudaSuccess ||
+                (e = cudaEventCreateWithFlags(&s->ev_out[b], cudaEventDisableTiming)) != cudaSuccess)
+                return cuda_fail(e, "event creation");
+    }
+    if (s->stage_bytes < 2 * per_set) {
         if (s->stage) {
-            if ((e = cudaStreamSynchronize(s->cs)) != cudaSuccess) return cuda_fail(e, "sync");
+            if ((e = cudaDeviceSynchronize()) != cudaSuccess) return cuda_fail(e, "sync");
             cudaFree(s->stage);
             s->stage = nullptr;
             s->stage_bytes = 0;
         }
-        if ((e = cudaMalloc(&s->stage, need)) != cudaSuccess) return cuda_fail(e, "staging");
-        s->stage_bytes = need;
+        if ((e = cudaMalloc(&s->stage, 2 * per_set)) != cudaSuccess)
+            return cuda_fail(e, "staging");
+        s->stage_bytes = 2 * per_set;
     }
-    uint8_t* base = static_cast<uint8_t*>(s->stage);
+    const int b = s->stage_turn;
+    uint8_t* base = static_cast<uint8_t*>(s->stage) + size_t(b) * per_set;
     void* dq = base;
     void* dk = base + in_bytes;
     void* dv = base + 2 * in_bytes;
     void* dout = base + 3 * in_bytes;
-    if ((e = cudaMemcpyAsync(dq, q_host, in_bytes, cudaMemcpyHostToDevice, s->cs)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(dk, k_host, in_bytes, cudaMemcpyHostToDevice, s->cs)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(dv, v_host, in_bytes, cudaMemcpyHostToDevice, s->cs)) != cudaSuccess)
+    if ((e = cudaStreamWaitEvent(s->cp_in, s->ev_done[b], 0)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(dk, k_host, in_bytes, cudaMemcpyHostToDevice, s->cp_in)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(dv, v_host, in_bytes, cudaMemcpyHostToDevice, s->cp_in)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(dq, q_host, in_bytes, cudaMemcpyHostToDevice, s->cp_in)) != cudaSuccess ||
+        (e = cudaEventRecord(s->ev_in[b], s->cp_in)) != cudaSuccess ||
+        (e = cudaStreamWaitEvent(s->cs, s->ev_in[b], 0)) != cudaSuccess ||
+        (e = cudaStreamWaitEvent(s->cs, s->ev_out[b], 0)) != cudaSuccess)
         return cuda_fail(e, "host-to-device copy");
     if ((st = frt_chunk_step(s, dq, dk, dv, dout, slot_out, evicted_out)) != FRT_OK) return st;
-    if ((e = cudaMemcpyAsync(out_host, dout, out_bytes, cudaMemcpyDeviceToHost, s->cs)) !=
-        cudaSuccess)
+    if ((e = cudaEventRecord(s->ev_done[b], s->cs)) != cudaSuccess ||
+        (e = cudaStreamWaitEvent(s->cp_out, s->ev_done[b], 0)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(out_host, dout, out_bytes, cudaMemcpyDeviceToHost, s->cp_out)) !=
+            cudaSuccess ||
+        (e = cudaEventRecord(s->ev_out[b], s->cp_out)) != cudaSuccess)
         return cuda_fail(e, "device-to-host copy");
+    s->stage_turn ^= 1;
     return FRT_OK;
 }
 
@@ -658,6 +710,8 @@ frt_status frt_stream_sync(frt_stream_t* s) {
     if (!s) return fail(FRT_ERR_INVALID_ARG, "NULL stream handle");
     if (!s->configured) return FRT_OK;
     cudaError_t e = cudaStreamSynchronize(s->cs);
+    if (e == cudaSuccess && s->cp_in) e = cudaStreamSynchronize(s->cp_in);
+    if (e == cudaSuccess && s->cp_out) e = cudaStreamSynchronize(s->cp_out);
     if (e != cudaSuccess) return cuda_fail(e, "stream sync");
     return check_device_status(s);
 }
@@ -666,6 +720,8 @@ frt_status frt_stream_reset(frt_stream_t* s) {
     if (!s) return fail(FRT_ERR_INVALID_ARG, "NULL stream handle");
     if (!s->configured) return fail(FRT_ERR_STATE, "stream not configured");
     cudaError_t e = cudaStreamSynchronize(s->cs);
+    if (e == cudaSuccess && s->cp_in) e = cudaStreamSynchronize(s->cp_in);
+    if (e == cudaSuccess && s->cp_out) e = cudaStreamSynchronize(s->cp_out);
     if (e != cudaSuccess) return cuda_fail(e, "stream sync");
     const size_t cache_bytes = size_t(s->window) * s->chunk_elems * 2;
     if ((e = cudaMemsetAsync(s->cache_k, 0, cache_bytes, s->cs)) != cudaSuccess ||

@@ -44,8 +44,11 @@ __device__ __forceinline__ uint32_t rope_pair(uint32_t x, float c, float s) {
     return r;
 }
 
-__device__ __forceinline__ float2 rope_cs(const RopeArgs& a, int pi, int f, int r, int col) {
-    if (pi < a.dt2) return a.t_tab[f * a.dt2 + pi];
+// t_tab: the chunk's t-segment table, either a.t_tab itself (parameter space) or a
+// shared-memory copy of it (kernels whose lanes index it divergently).
+__device__ __forceinline__ float2 rope_cs(const RopeArgs& a, const float2* t_tab, int pi, int f,
+                                          int r, int col) {
+    if (pi < a.dt2) return t_tab[f * a.dt2 + pi];
     pi -= a.dt2;
     if (pi < a.dh2) return a.hw[r * a.dh2 + pi];
     pi -= a.dh2;
@@ -55,13 +58,13 @@ __device__ __forceinline__ float2 rope_cs(const RopeArgs& a, int pi, int f, int 
 // Rotate 8 consecutive head_dim elements [d0, d0+8) (d0 % 8 == 0) of a token at
 // frame f, row r, column col.
 __device__ __forceinline__ uint4 rope_rotate8(uint4 v, int d0, int f, int r, int col,
-                                              const RopeArgs& a) {
+                                              const RopeArgs& a, const float2* t_tab) {
     const int p0 = d0 >> 1;
     float2 cs;
-    cs = rope_cs(a, p0 + 0, f, r, col); v.x = rope_pair(v.x, cs.x, cs.y);
-    cs = rope_cs(a, p0 + 1, f, r, col); v.y = rope_pair(v.y, cs.x, cs.y);
-    cs = rope_cs(a, p0 + 2, f, r, col); v.z = rope_pair(v.z, cs.x, cs.y);
-    cs = rope_cs(a, p0 + 3, f, r, col); v.w = rope_pair(v.w, cs.x, cs.y);
+    cs = rope_cs(a, t_tab, p0 + 0, f, r, col); v.x = rope_pair(v.x, cs.x, cs.y);
+    cs = rope_cs(a, t_tab, p0 + 1, f, r, col); v.y = rope_pair(v.y, cs.x, cs.y);
+    cs = rope_cs(a, t_tab, p0 + 2, f, r, col); v.z = rope_pair(v.z, cs.x, cs.y);
+    cs = rope_cs(a, t_tab, p0 + 3, f, r, col); v.w = rope_pair(v.w, cs.x, cs.y);
     return v;
 }
 
@@ -109,6 +112,7 @@ struct AppendParams {
     int vec_per_tok;        // H * D / 8
     int vec_per_head_log2;  // log2(D / 8)
     int rope;               // rotate K on the way
+    DeviceStatus* status;   // bounded-wait timeouts are recorded here
     RopeArgs ra;
 };
 
@@ -118,6 +122,7 @@ struct RopeParams {
     int n_tok;
     int vec_per_tok;
     int vec_per_head_log2;
+    DeviceStatus* status;
     RopeArgs ra;
 };
 
