@@ -22,9 +22,9 @@
 // in issue order, so S_g(j+1) never overwrites P_g(j) early, and the arrival of S_g(j)
 // implies PV_g(j-1) is complete (so O_g may be rescaled then). While one tile's softmax
 // runs, the tensor pipe works on the other tile's PV and next S.
-// The softmax keeps a running max in the log2 domain and rescales O only when the row
-// max grows by more than 2^kRescaleLog2 (O and the row sum share the stale max, so the
-// result is exact).
+// The softmax exponentiates against a stale reference max in the log2 domain and
+// rescales O only when a row's sum signals possible overflow (O and the row sum share
+// the reference, so the result is exact).
 //
 // Every wait is bounded (mbar_wait): a role that gives up records FRT_ERR_TIMEOUT in the
 // stream's status block, raises a CTA-wide abort flag, and the CTA drains its in-flight
@@ -45,7 +45,7 @@ constexpr int kRegsSm = 200;
 static_assert(128 * kRegsCtl + 256 * kRegsSm == kThreads * kRegsLaunch, "register split");
 constexpr int kBM = 128;   // query rows per tile
 constexpr int kBN = 128;   // KV rows per tile
-constexpr float kRescaleLog2 = 8.0f;
+constexpr float kOverflowGuard = 1.152921504606846976e18f;   // 2^60
 constexpr int kTimeoutCode = 6;  // FRT_ERR_TIMEOUT
 
 template <int D>
@@ -276,35 +276,35 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 else ok = wait_load(1);
                 umma_commit(smem_u32(&bars->kv_empty[0]));
             }
+            // ring slots of the previous step (V_{j-1}, K_j) are released from inside the
+            // first MMA group of step j, off the loop's critical path (a commit tracks
+            // every earlier MMA, so releasing one MMA later is still correct)
+            int prev_sv = -1, prev_sk = -1;
             for (int j = 0; j < n_tiles && ok; ++j) {
                 const bool more = (j + 1) < n_tiles;
                 const int sv = (2 * j + 1) % C::STAGES, sk = (2 * j + 2) % C::STAGES;
                 // V_j has been waited for; K_{j+1} is waited for inside PV_0(j);
                 // V_{j+1} inside the last group of this step.
                 if (!(ok = wait_p(0, j))) break;
-                issue_o(0, sv, j > 0, [&] { if (more) ok = wait_load(2 * j + 2); });
+                issue_o(0, sv, j > 0, [&] {
+                    if (prev_sv >= 0) umma_commit(smem_u32(&bars->kv_empty[prev_sv]));
+                    if (prev_sk >= 0) umma_commit(smem_u32(&bars->kv_empty[prev_sk]));
+                    if (more) ok = wait_load(2 * j + 2);
+                });
                 if (!ok) break;
                 if (ng == 2) {
                     if (more) issue_s(0, sk, nop);
                     else umma_commit(smem_u32(&bars->o_done[0]));
                     if (!(ok = wait_p(1, j))) break;
                     issue_o(1, sv, j > 0, nop);
-                    umma_commit(smem_u32(&bars->kv_empty[sv]));
-                    if (more) {
-                        issue_s(1, sk, [&] { ok = wait_load(2 * j + 3); });
-                        umma_commit(smem_u32(&bars->kv_empty[sk]));
-                    } else {
-                        umma_commit(smem_u32(&bars->o_done[1]));
-                    }
+                    if (more) issue_s(1, sk, [&] { ok = wait_load(2 * j + 3); });
+                    else umma_commit(smem_u32(&bars->o_done[1]));
                 } else {
-                    umma_commit(smem_u32(&bars->kv_empty[sv]));
-                    if (more) {
-                        issue_s(0, sk, [&] { ok = wait_load(2 * j + 3); });
-                        umma_commit(smem_u32(&bars->kv_empty[sk]));
-                    } else {
-                        umma_commit(smem_u32(&bars->o_done[0]));
-                    }
+                    if (more) issue_s(0, sk, [&] { ok = wait_load(2 * j + 3); });
+                    else umma_commit(smem_u32(&bars->o_done[0]));
                 }
+                prev_sv = sv;
+                prev_sk = more ? sk : -1;
             }
             // drain: all issued MMAs complete before TMEM is released
             umma_commit(smem_u32(&bars->drain[0]));
@@ -370,13 +370,15 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 for (int i = 0; i < kBN; ++i)
                     if (i >= valid) s[i] = -INFINITY;
             }
-            // The exponentials of the first 64 scores are computed against the running
-            // (stale) max at the same time as the row max: they only have to be redone
-            // when the max grows by more than 2^kRescaleLog2, which after the first few
-            // tiles is rare. This keeps the max reduction off the critical path.
+            // p = 2^(s * scale * log2 e - m) against a reference m that is the exact row
+            // max only on the first tile; afterwards it is left stale. bf16 P shares
+            // fp32's exponent range, so stale values are harmless until a p could
+            // overflow: every p is bounded by the row sum, so a row sum above
+            // kOverflowGuard (rare) triggers the exact max, a rescale of O and a redo.
+            // No row-max reduction runs on the common path.
             const uint64_t sl2x2 = f2_pack(sl2, sl2);
             uint32_t pk[32];
-            uint64_t acc[4] = {0, 0, 0, 0};
+            uint64_t acc[4];
             auto exp_half = [&](int h, float mref) {
                 const uint64_t negm = f2_pack(-mref, -mref);
 #pragma unroll
@@ -390,26 +392,43 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                     pk[i] = pack_bf16x2(p0, p1);
                 }
             };
-            if (j > 0) exp_half(0, m_run);
-            // row max: 8 independent 3-input max chains
-            float mx[8];
+            auto exp_row = [&](float mref) {
+                acc[0] = acc[1] = acc[2] = acc[3] = 0;
+                exp_half(0, mref);
+                tmem_st32(tS, pk);
+                exp_half(1, mref);
+                tmem_st32(tS + 32, pk);
+            };
+            auto row_max = [&]() -> float {   // 8 independent 3-input max chains
+                float mx[8];
 #pragma unroll
-            for (int a = 0; a < 8; ++a) mx[a] = fmaxf(s[a], s[a + 8]);
+                for (int a = 0; a < 8; ++a) mx[a] = fmaxf(s[a], s[a + 8]);
 #pragma unroll
-            for (int i = 16; i < kBN; i += 16)
+                for (int i = 16; i < kBN; i += 16)
 #pragma unroll
-                for (int a = 0; a < 8; ++a) mx[a] = max3f(mx[a], s[i + a], s[i + 8 + a]);
-            const float mrow = max3f(max3f(mx[0], mx[1], mx[2]), max3f(mx[3], mx[4], mx[5]),
-                                     fmaxf(mx[6], mx[7]));
-            const float m_new = fmaxf(m_run, mrow * sl2);
-            const bool need = m_new > m_run + kRescaleLog2;
+                    for (int a = 0; a < 8; ++a) mx[a] = max3f(mx[a], s[i + a], s[i + 8 + a]);
+                return max3f(max3f(mx[0], mx[1], mx[2]), max3f(mx[3], mx[4], mx[5]),
+                             fmaxf(mx[6], mx[7]));
+            };
+            auto row_sum = [&]() -> float {
+                float a0, a1, b0, b1, c0, c1, d0, d1;
+                f2_unpack(acc[0], a0, a1);
+                f2_unpack(acc[1], b0, b1);
+                f2_unpack(acc[2], c0, c1);
+                f2_unpack(acc[3], d0, d1);
+                return ((a0 + a1) + (b0 + b1)) + ((c0 + c1) + (d0 + d1));
+            };
             float alpha = 1.0f;
-            if (need) {
-                alpha = ex2_approx(m_run - m_new);
-                m_run = m_new;
-            }
-            if (j == 0 || __any_sync(0xffffffffu, need)) {
-                if (j > 0) {
+            if (j == 0) {
+                m_run = row_max() * sl2;
+                exp_row(m_run);
+            } else {
+                exp_row(m_run);
+                const bool big = row_sum() > kOverflowGuard;
+                if (__any_sync(0xffffffffu, big)) {
+                    const float m_new = fmaxf(m_run, row_max() * sl2);
+                    alpha = ex2_approx(m_run - m_new);
+                    m_run = m_new;
                     // S_g(j) has landed, so PV_g(j-1) is complete: O_g is stable
 #pragma unroll 1
                     for (int c = 0; c < D / 32; ++c) {
@@ -428,19 +447,11 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                         }
                         tmem_st32(tO + c * 32, o);
                     }
+                    tmem_st_wait();   // the first P stores complete before they are replaced
+                    exp_row(m_run);
                 }
-                acc[0] = acc[1] = acc[2] = acc[3] = 0;
-                exp_half(0, m_run);
             }
-            tmem_st32(tS, pk);
-            exp_half(1, m_run);
-            tmem_st32(tS + 32, pk);
-            float a0, a1, b0, b1, c0, c1, d0, d1;
-            f2_unpack(acc[0], a0, a1);
-            f2_unpack(acc[1], b0, b1);
-            f2_unpack(acc[2], c0, c1);
-            f2_unpack(acc[3], d0, d1);
-            l_run = l_run * alpha + (((a0 + a1) + (b0 + b1)) + ((c0 + c1) + (d0 + d1)));
+            l_run = l_run * alpha + row_sum();
             tmem_st_wait();
             tc_fence_before();
             mbar_arrive(smem_u32(&bars->p_full[g]));

@@ -181,3 +181,28 @@ def test_host_buffer_step_pipelined_matches_device_path_and_oracle(frt):
         assert np.array_equal(got, dev[c][0]), c
         U.assert_close(got, ref[c][0], f"host path chunk {c}")
     a.close(); b.close()
+
+
+@pytest.mark.parametrize("scale_last", [20.0, 0.05])
+def test_scores_growing_or_shrinking_across_tiles(frt, scale_last):
+    """Keys of the newest chunk scaled up (scores far above every earlier tile: the
+    kernel's stale exponent reference must be replaced and O rescaled) or down (later
+    tiles far below the reference): the result still matches the oracle."""
+    from oracle.frt_oracle import OracleStream
+    wl = SMALL["ragged_d128"]
+    st = U.make_stream(wl, frt)
+    orc = OracleStream(wl.heads, wl.head_dim, wl.grid_h, wl.grid_w, wl.frames, wl.window,
+                       wl.split)
+    for c in range(wl.window):
+        q, k, v = synth.chunk_qkv(wl, 0, c)
+        if c == wl.window - 1:
+            k = (k.float() * scale_last).to(torch.bfloat16)
+        ref = orc.step(synth.as_f64(q), synth.as_f64(k), synth.as_f64(v))[0]
+        qd, kd, vd = q.cuda(), k.cuda(), v.cuda()
+        out = st.new_out()
+        st.chunk_step(qd, kd, vd, out)
+        st.sync()
+        got = out.cpu().numpy()
+        assert np.all(np.isfinite(got))
+        U.assert_close(got, ref, f"chunk {c} scale {scale_last}")
+    st.close()
