@@ -280,9 +280,9 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             // first MMA group of step j, off the loop's critical path (a commit tracks
             // every earlier MMA, so releasing one MMA later is still correct)
             int prev_sv = -1, prev_sk = -1;
+            int sv = 1 % C::STAGES, sk = 2 % C::STAGES;   // ring slots of V_j and K_{j+1}
             for (int j = 0; j < n_tiles && ok; ++j) {
                 const bool more = (j + 1) < n_tiles;
-                const int sv = (2 * j + 1) % C::STAGES, sk = (2 * j + 2) % C::STAGES;
                 // V_j has been waited for; K_{j+1} is waited for inside PV_0(j);
                 // V_{j+1} inside the last group of this step.
                 if (!(ok = wait_p(0, j))) break;
@@ -305,6 +305,8 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 }
                 prev_sv = sv;
                 prev_sk = more ? sk : -1;
+                sv = (sv + 2 >= C::STAGES) ? sv + 2 - C::STAGES : sv + 2;
+                sk = (sk + 2 >= C::STAGES) ? sk + 2 - C::STAGES : sk + 2;
             }
             // drain: all issued MMAs complete before TMEM is released
             umma_commit(smem_u32(&bars->drain[0]));
