@@ -22,6 +22,17 @@ extern "C" {
 int frt_selftest_umma_tile(const void* a, const void* b, float* c, int b_mn_major, int lbo_b,
                            int sbo_b, int a_from_tmem, int* dev_status, void* cuda_stream);
 
+/* A CTA pair (cluster of 2) computes one 256x128x128 bf16 tile C = A B^T with
+ * tcgen05.mma.cta_group::2: CTA r loads rows [128r, 128r+128) of A and rows
+ * [64r, 64r+64) of B with TMA (completion signalled on the leader CTA's mbarrier),
+ * the leader issues the MMAs, each CTA reads its 128 rows of D from its TMEM.
+ *   a: device [256, 128] bf16 row-major; b: device [128, 128] bf16 row-major (b[n][k]);
+ *   c: device [256, 128] fp32; taddrs: device uint32[2], the TMEM address each CTA got
+ *   from the pair allocation; dev_status: device int set to 1 on a timeout.
+ * Returns 0 on launch success, < 0 on an argument/launch error. */
+int frt_selftest_umma_pair(const void* a, const void* b, float* c, unsigned* taddrs,
+                           int* dev_status, void* cuda_stream);
+
 /* Launch a kernel whose one waiting thread waits on an mbarrier that nothing arrives
  * on, bounded by limit_ns (<= 100 ms); it must record FRT_ERR_TIMEOUT in s's status
  * block, which frt_stream_sync then returns. s must be configured. */

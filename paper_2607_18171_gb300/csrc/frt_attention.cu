@@ -70,7 +70,8 @@ struct Bars {
     uint64_t o_done[2];
     uint64_t drain[2];
     uint64_t kv_full[8];
-    uint64_t kv_empty[8];
+    uint64_t step_done[4];
+    uint64_t k0_done;
     uint32_t tmem_base;
     int abort_flag;
     int last_split;
@@ -154,7 +155,8 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
         mbar_init(smem_u32(&bars->drain[1]), 1);
         for (int s = 0; s < C::STAGES; ++s) {
             mbar_init(smem_u32(&bars->kv_full[s]), 1);
-            mbar_init(smem_u32(&bars->kv_empty[s]), 1);
+        for (int s = 0; s < 4; ++s) mbar_init(smem_u32(&bars->step_done[s]), 1);
+        mbar_init(smem_u32(&bars->k0_done), 1);
         }
         bars->abort_flag = 0;
         fence_mbar_init();
@@ -184,14 +186,28 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 for (int cb = 0; cb < C::NCB; ++cb)
                     tma_load_3d(sQ + g * C::Q_TILE + cb * (kBM * 128), &sd.q_map, qbar,
                                 cb * 64, head, m0 + g * kBM);
+            // Load L reuses the ring slot of load L - STAGES. Slots are released per KV
+            // step: step j reads V_j and K_{j+1} (loads 2j+1, 2j+2) and its single release
+            // commit arrives on step_done[j % 4]; K_0 (load 0) is released by k0_done.
+            // Step j+4 needs loads the producer has not issued while it waits for step
+            // j, so the parity of step_done[j % 4] is never ambiguous.
             int L = 0;
             for (; L < n_loads; ++L) {
                 const int stage = L % C::STAGES;
-                const int round = L / C::STAGES;
-                if (round > 0 &&
-                    !mbar_wait(smem_u32(&bars->kv_empty[stage]), (round - 1) & 1, lim, abort)) {
-                    report(p.status, abort, 0, L);
-                    break;
+                if (L >= C::STAGES) {
+                    const int prev = L - C::STAGES;
+                    bool got;
+                    if (prev == 0) {
+                        got = mbar_wait(smem_u32(&bars->k0_done), 0, lim, abort);
+                    } else {
+                        const int step = (prev - 1) >> 1;
+                        got = mbar_wait(smem_u32(&bars->step_done[step & 3]), (step >> 2) & 1,
+                                        lim, abort);
+                    }
+                    if (!got) {
+                        report(p.status, abort, 0, L);
+                        break;
+                    }
                 }
                 const CUtensorMap* map = (L & 1) ? &sd.v_map : &sd.k_map;
                 const int row = (t0 + (L >> 1)) * kBN;
@@ -235,8 +251,9 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 return true;
             };
             // MMA groups: S_g = Q_g K^T (8 MMAs over D) and O_g += P_g V (8 MMAs over the
-            // KV tile). `mid` runs after the first MMA of a group, while the tensor pipe
-            // still has work queued: waits for loads needed later are hidden there.
+            // KV tile). `mid(k)` runs after MMA k of a group, while the tensor pipe still
+            // works on it: after issuing an MMA the thread has about one MMA (64 cycles) of
+            // slack, so bookkeeping is spread one operation per gap to stay hidden.
             auto issue_s = [&](int g, int stage, auto&& mid) {
                 const uint64_t dq = dq0 + uint64_t((g * C::Q_TILE) >> 4);
                 const uint64_t dk = dk0 + uint64_t((stage * C::KV_TILE) >> 4);
@@ -245,7 +262,7 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 for (int k = 0; k < D / 16; ++k) {
                     const uint64_t off = uint64_t((k >> 2) * ((kBM * 128) >> 4) + (k & 3) * 2);
                     umma_ss(d, dq + off, dk + off, C::IDESC_S, k > 0 ? 1u : 0u);
-                    if (k == 0) mid();
+                    mid(k);
                 }
                 umma_commit(smem_u32(&bars->s_full[g]));
             };
@@ -257,7 +274,7 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 for (int k = 0; k < kBN / 16; ++k) {
                     umma_ts(d, pa + k * 8, dv + uint64_t(k * ((16 * 128) >> 4)), C::IDESC_O,
                             (acc || k > 0) ? 1u : 0u);
-                    if (k == 0) mid();
+                    mid(k);
                 }
             };
             auto wait_p = [&](int g, int j) -> bool {
@@ -268,43 +285,35 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 tc_fence_after();
                 return true;
             };
-            auto nop = [] {};
+            auto nop = [](int) {};
             // load order of the producer: K0, V0, K1, V1, ... -> load 2j is K_j, 2j+1 is V_j
             if (ok && (ok = wait_load(0))) {
                 issue_s(0, 0, nop);
-                if (ng == 2) issue_s(1, 0, [&] { ok = wait_load(1); });
+                if (ng == 2) issue_s(1, 0, [&](int k) { if (k == 0) ok = wait_load(1); });
                 else ok = wait_load(1);
-                umma_commit(smem_u32(&bars->kv_empty[0]));
+                umma_commit(smem_u32(&bars->k0_done));
             }
-            // ring slots of the previous step (V_{j-1}, K_j) are released from inside the
-            // first MMA group of step j, off the loop's critical path (a commit tracks
-            // every earlier MMA, so releasing one MMA later is still correct)
-            int prev_sv = -1, prev_sk = -1;
             int sv = 1 % C::STAGES, sk = 2 % C::STAGES;   // ring slots of V_j and K_{j+1}
             for (int j = 0; j < n_tiles && ok; ++j) {
                 const bool more = (j + 1) < n_tiles;
                 // V_j has been waited for; K_{j+1} is waited for inside PV_0(j);
                 // V_{j+1} inside the last group of this step.
                 if (!(ok = wait_p(0, j))) break;
-                issue_o(0, sv, j > 0, [&] {
-                    if (prev_sv >= 0) umma_commit(smem_u32(&bars->kv_empty[prev_sv]));
-                    if (prev_sk >= 0) umma_commit(smem_u32(&bars->kv_empty[prev_sk]));
-                    if (more) ok = wait_load(2 * j + 2);
-                });
+                issue_o(0, sv, j > 0, [&](int k) { if (k == 0 && more) ok = wait_load(2 * j + 2); });
                 if (!ok) break;
                 if (ng == 2) {
                     if (more) issue_s(0, sk, nop);
                     else umma_commit(smem_u32(&bars->o_done[0]));
                     if (!(ok = wait_p(1, j))) break;
                     issue_o(1, sv, j > 0, nop);
-                    if (more) issue_s(1, sk, [&] { ok = wait_load(2 * j + 3); });
+                    if (more) issue_s(1, sk, [&](int k) { if (k == 0) ok = wait_load(2 * j + 3); });
                     else umma_commit(smem_u32(&bars->o_done[1]));
+                    if (more) umma_commit(smem_u32(&bars->step_done[j & 3]));
                 } else {
-                    if (more) issue_s(0, sk, [&] { ok = wait_load(2 * j + 3); });
+                    if (more) issue_s(0, sk, [&](int k) { if (k == 0) ok = wait_load(2 * j + 3); });
                     else umma_commit(smem_u32(&bars->o_done[0]));
+                    if (more) umma_commit(smem_u32(&bars->step_done[j & 3]));
                 }
-                prev_sv = sv;
-                prev_sk = more ? sk : -1;
                 sv = (sv + 2 >= C::STAGES) ? sv + 2 - C::STAGES : sv + 2;
                 sk = (sk + 2 >= C::STAGES) ? sk + 2 - C::STAGES : sk + 2;
             }

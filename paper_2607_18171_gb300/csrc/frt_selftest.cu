@@ -123,6 +123,86 @@ umma_tile_kernel(const __grid_constant__ CUtensorMap a_map, const __grid_constan
     if (warp == 0) tmem_dealloc(tmem, 256);
 }
 
+// ----------------------------------------------------------------------------------------
+// CTA pair: one M=256 x N=128 x K=128 tile with tcgen05.mma.cta_group::2. CTA r of the
+// pair holds rows [128 r, 128 r + 128) of A and rows [64 r, 64 r + 64) of B (the N
+// half); the leader (rank 0) issues the MMAs; each CTA reads its 128 rows of D.
+// ----------------------------------------------------------------------------------------
+constexpr int kPairA = 128 * 128 * 2;
+constexpr int kPairB = 64 * 128 * 2;
+constexpr int kPairSmem = kPairA + kPairB + 1024;
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(128, 1)
+umma_pair_kernel(const __grid_constant__ CUtensorMap a_map, const __grid_constant__ CUtensorMap b_map,
+                 float* c, uint32_t* taddrs, int* status) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~uintptr_t(1023));
+    const uint32_t sA = smem_u32(smem), sB = sA + kPairA;
+    __shared__ uint64_t full, done;
+    __shared__ uint32_t tbase;
+    __shared__ int abort_flag;
+    const uint32_t rank = cluster_ctarank();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint64_t lim = 1000000000ull;
+    if (threadIdx.x == 0) {
+        mbar_init(smem_u32(&full), 1);
+        mbar_init(smem_u32(&done), 1);
+        abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tmem_alloc_pair(smem_u32(&tbase), 256);
+        tmem_relinquish_pair();
+    }
+    tc_fence_before();
+    cluster_sync_all();
+    tc_fence_after();
+    const uint32_t tmem = tbase;
+    if (threadIdx.x == 0) taddrs[rank] = tmem;
+    if (threadIdx.x == 0) {
+        const uint32_t full_leader = mapa_shared(smem_u32(&full), 0);
+        if (rank == 0) mbar_arrive_expect_tx(smem_u32(&full), 2 * (kPairA + kPairB));
+        for (int cb = 0; cb < 2; ++cb) {
+            tma_load_2d_pair(sA + cb * (128 * 128), &a_map, full_leader, cb * 64, int(rank) * 128);
+            tma_load_2d_pair(sB + cb * (64 * 128), &b_map, full_leader, cb * 64, int(rank) * 64);
+        }
+        if (rank == 0) {
+            if (mbar_wait(smem_u32(&full), 0, lim, &abort_flag)) {
+                tc_fence_after();
+                const uint32_t idesc = idesc_bf16_f32(256, 128, false);
+                for (int k = 0; k < 8; ++k) {
+                    const uint32_t aoff = (k >> 2) * (128 * 128) + (k & 3) * 32;
+                    const uint32_t boff = (k >> 2) * (64 * 128) + (k & 3) * 32;
+                    umma_ss_pair(tmem, sdesc_sw128(sA + aoff, 16, 1024),
+                                 sdesc_sw128(sB + boff, 16, 1024), idesc, k > 0);
+                }
+                umma_commit_pair(smem_u32(&done), 0x3);
+            }
+        }
+    }
+    bool ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&done), 0, lim, &abort_flag));
+    if (ok) {
+        tc_fence_after();
+        const int row = warp * 32 + lane;
+        const uint32_t lane_off = uint32_t(warp * 32) << 16;
+        for (int cc = 0; cc < 4; ++cc) {
+            uint32_t r[32];
+            tmem_ld32(tmem + lane_off + cc * 32, r);
+            tmem_ld_wait();
+            for (int i = 0; i < 32; ++i)
+                c[(size_t(rank) * 128 + row) * 128 + cc * 32 + i] = __uint_as_float(r[i]);
+        }
+    } else if (lane == 0) {
+        atomicExch(status, 1);
+    }
+    // both CTAs are done with TMEM and with each other's shared memory
+    tc_fence_before();
+    cluster_sync_all();
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc_pair(tmem, 256);
+}
+
 __global__ void wait_timeout_kernel(DeviceStatus* st, unsigned long long limit_ns) {
     __shared__ uint64_t bar;
     __shared__ int abort_flag;
@@ -150,6 +230,25 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+int map_2d(CUtensorMap* m, const void* ptr, int rows, int box_rows) {
+    void* fp = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fp, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+        return 1;
+    auto fn = reinterpret_cast<EncodeTiledFn>(fp);
+    cuuint64_t dims[2] = {128, cuuint64_t(rows)};
+    cuuint64_t strides[1] = {256};
+    cuuint32_t box[2] = {64, cuuint32_t(box_rows)};
+    cuuint32_t es[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box,
+              es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS
+               ? 0
+               : 2;
+}
 
 int map_128x128(CUtensorMap* m, const void* ptr) {
     void* fp = nullptr;
@@ -186,6 +285,19 @@ extern "C" int frt_selftest_umma_tile(const void* a, const void* b, float* c, in
         return -3;
     umma_tile_kernel<<<1, 128, kSmem, st>>>(am, bm, c, b_mn_major, lbo_b, sbo_b, a_from_tmem,
                                             dev_status);
+    return cudaGetLastError() == cudaSuccess ? 0 : -4;
+}
+
+extern "C" int frt_selftest_umma_pair(const void* a, const void* b, float* c, unsigned* taddrs,
+                                      int* dev_status, void* cuda_stream) {
+    if (!a || !b || !c || !taddrs || !dev_status) return -1;
+    CUtensorMap am, bm;
+    if (map_2d(&am, a, 256, 128) || map_2d(&bm, b, 128, 64)) return -2;
+    if (cudaFuncSetAttribute(umma_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             kPairSmem) != cudaSuccess)
+        return -3;
+    umma_pair_kernel<<<2, 128, kPairSmem, static_cast<cudaStream_t>(cuda_stream)>>>(
+        am, bm, c, taddrs, dev_status);
     return cudaGetLastError() == cudaSuccess ? 0 : -4;
 }
 

@@ -73,6 +73,7 @@ def lib() -> ctypes.CDLL:
         "frt_version": (ctypes.c_char_p, []),
         "frt_selftest_umma_tile": (I, [P, P, P, I, I, I, I, P, P]),
         "frt_selftest_wait_timeout": (I, [P, LL, P]),
+        "frt_selftest_umma_pair": (I, [P, P, P, P, P, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -273,6 +274,21 @@ def selftest_umma_tile(a: torch.Tensor, b: torch.Tensor, b_mn_major: bool, lbo: 
     if int(status.item()) != 0:
         raise FrtError(6, "selftest tile timed out")
     return c
+
+
+def selftest_umma_pair(a: torch.Tensor, b: torch.Tensor):
+    """(C [256,128] fp32, TMEM addresses the two CTAs got) for C = A B^T on a CTA pair."""
+    c = torch.empty(256, 128, dtype=torch.float32, device="cuda")
+    taddrs = torch.zeros(2, dtype=torch.int32, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    rc = lib().frt_selftest_umma_pair(_ptr(a), _ptr(b), _ptr(c), _ptr(taddrs), _ptr(status),
+                                      ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+    if rc != 0:
+        raise FrtError(4, f"pair selftest launch failed ({rc})")
+    torch.cuda.synchronize()
+    if int(status.item()) != 0:
+        raise FrtError(6, "pair selftest timed out")
+    return c, taddrs.cpu().tolist()
 
 
 def selftest_wait_timeout(stream: Stream, limit_ns: int) -> None:

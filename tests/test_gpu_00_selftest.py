@@ -65,3 +65,13 @@ def test_bounded_wait_reports_timeout_and_context_survives(frt):
     st.sync()
     assert torch.isfinite(out).all()
     st.close()
+
+
+def test_umma_cta_pair_tile(frt):
+    """tcgen05.mma.cta_group::2 on a CTA pair: A rows split across the CTAs, B split by N."""
+    g = torch.Generator().manual_seed(4)
+    a = torch.randn(256, 128, generator=g).to(torch.bfloat16)
+    b = torch.randn(128, 128, generator=g).to(torch.bfloat16)
+    c, taddrs = frt.selftest_umma_pair(a.cuda(), b.cuda())
+    assert taddrs[0] == taddrs[1]      # one allocation shared by the pair
+    _check(c, a.double() @ b.double().T)
