@@ -166,6 +166,8 @@ def run_gpu(args, wl, world, rank, local):
 
     if wl.streams > 1:
         return run_gpu_multi(args, wl, world, rank, local, dev, peak_tf, peak_kind)
+    if wl.steps > 1:
+        return run_gpu_steps(args, wl, world, rank, local, dev, peak_tf, peak_kind)
 
     sid = rank  # each rank streams its own independent video (weak scaling)
     st = frt.Stream(wl.heads, wl.head_dim, wl.grid_h, wl.grid_w, wl.frames, wl.window,
@@ -345,6 +347,61 @@ def run_gpu_multi(args, wl, world, rank, local, dev, peak_tf, peak_kind):
                      "launch_ms": round(attn_mean, 4)},
         "clocks": clk.summary(),
         "gpu_launches": (2 * wl.streams + 1) * n,
+    }
+
+
+def run_gpu_steps(args, wl, world, rank, local, dev, peak_tf, peak_kind):
+    """Per-denoising-step caches: every tick advances all wl.steps steps by one chunk
+    (RoPE + append per step) and runs one batched attention over them, at steady
+    state (full windows)."""
+    import torch
+    from paper_2607_18171_gb300 import frt, synth
+
+    stream = torch.cuda.current_stream()
+    grp = frt.Steps(wl.steps, wl.heads, wl.head_dim, wl.grid_h, wl.grid_w, wl.frames,
+                    wl.window, split=wl.split)
+    sets = [[tuple(t.to(dev) for t in synth.chunk_qkv(wl, 100 * rank + i, 50 + r))
+             for i in range(wl.steps)] for r in range(2)]
+    outs = {i: torch.empty(grp.shape(), dtype=torch.float32, device=dev)
+            for i in range(wl.steps)}
+    act = list(range(wl.steps))
+
+    def tick(t):
+        w = sets[t % 2]
+        grp.tick(act, {i: w[i][0] for i in act}, {i: w[i][1] for i in act},
+                 {i: w[i][2] for i in act}, outs)
+
+    for t in range(wl.window - 1 + args.warmup):   # fill every window, then warm up
+        tick(t)
+    torch.cuda.synchronize()
+    n = args.steps
+    flops = wl.steps * wl.attn_flops(wl.window - 1)
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        t0.record(stream)
+        for t in range(n):
+            tick(t)
+        t1.record(stream)
+        torch.cuda.synchronize()
+    elapsed = max_over_ranks(t0.elapsed_time(t1), world, dev)
+    grp.close()
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    if rank != 0:
+        return None
+    return {
+        "metric": METRIC, "value": round(flops * n * world / (elapsed * 1e-3) / 1e12, 2),
+        "unit": UNIT, "n_gpus": world, "steps": n, "warmup": args.warmup,
+        "ms_per_step": round(elapsed / n, 4), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": describe(wl) + f", {wl.steps} denoising steps (own caches), "
+                   "one pipeline tick per step: RoPE + append per step, one batched attention",
+                   "note": "each tick re-rotates the same two input sets in place; timing only"},
+        "clocks": clk.summary(),
+        "gpu_launches": (2 * wl.steps + 1) * n,
     }
 
 

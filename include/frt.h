@@ -168,6 +168,28 @@ frt_status frt_chunk_attention_noalloc(const void* q, const void* k, const void*
                                        int head_dim, double sm_scale, int out_dtype,
                                        void* status, void* cuda_stream);
 
+/* Per-denoising-step caches. Each denoising step of the DiT keeps its own KV cache
+ * (section 3.1 "Case study"; Appendix A.4: step Q_i of batch j+1 depends only on
+ * step Q_i of batch j), which is what makes pipelining across steps legal. A step
+ * group owns n_steps independent streams of one shape; frt_steps_tick advances the
+ * active steps of one pipeline tick: in the wavefront schedule step i works on chunk
+ * t - i at tick t, so the steps' attentions are independent and run as ONE batched
+ * launch (the single-GPU form of the paper's stage pipeline over denoising steps).
+ * 1 <= n_steps <= 32; all steps share one frt_config (and CUDA stream). */
+typedef struct frt_steps frt_steps_t;
+frt_steps_t* frt_steps_create(int n_steps, int heads, int head_dim, int tokens_per_frame,
+                              int frames_per_chunk, int window_chunks);
+frt_status frt_steps_configure(frt_steps_t* g, const frt_config* cfg);
+/* The stream of step `step` (owned by the group; do not destroy it). NULL if out of range. */
+frt_stream_t* frt_steps_stream(const frt_steps_t* g, int step);
+/* One tick: for every step i with bit i of active_mask set, rotate q[i], k[i] in place
+ * (frt_rope3d_qk at that step's own chunk counter), append (k[i], v[i]) to its cache,
+ * then one batched attention launch writes out[i] for all active steps. Arrays are
+ * indexed by step; entries of inactive steps are ignored. */
+frt_status frt_steps_tick(frt_steps_t* g, unsigned int active_mask, void* const* q,
+                          void* const* k, const void* const* v, void* const* out);
+void frt_steps_destroy(frt_steps_t* g);
+
 /* Wait for the stream's work and return its device status (FRT_OK or the
  * first device error, e.g. FRT_ERR_TIMEOUT). */
 frt_status frt_stream_sync(frt_stream_t* s);

@@ -781,3 +781,81 @@ void frt::set_last_error(const char* msg) { g_last_error = msg; }
 extern "C" void* frt_internal_status_dev(frt_stream_t* s) {
     return (s && s->configured) ? static_cast<void*>(s->status_dev) : nullptr;
 }
+
+// ---------------------------------------------------------------------------------------
+// Per-denoising-step caches: a group of independent streams advanced by pipeline ticks.
+// ---------------------------------------------------------------------------------------
+struct frt_steps {
+    int n = 0;
+    frt_stream_t* st[kMaxBatchStreams] = {};
+};
+
+extern "C" {
+
+frt_steps_t* frt_steps_create(int n_steps, int heads, int head_dim, int tokens_per_frame,
+                              int frames_per_chunk, int window_chunks) {
+    if (n_steps < 1 || n_steps > kMaxBatchStreams) {
+        fail(FRT_ERR_INVALID_ARG, "1 <= n_steps <= %d", kMaxBatchStreams);
+        return nullptr;
+    }
+    frt_steps_t* g = new (std::nothrow) frt_steps();
+    if (!g) {
+        fail(FRT_ERR_OOM, "host allocation failed");
+        return nullptr;
+    }
+    for (int i = 0; i < n_steps; ++i) {
+        g->st[i] = frt_stream_create(heads, head_dim, tokens_per_frame, frames_per_chunk,
+                                     window_chunks);
+        if (!g->st[i]) {
+            frt_steps_destroy(g);
+            return nullptr;   // frt_last_error() set by frt_stream_create
+        }
+        g->n = i + 1;
+    }
+    return g;
+}
+
+frt_status frt_steps_configure(frt_steps_t* g, const frt_config* cfg) {
+    if (!g || !cfg) return fail(FRT_ERR_INVALID_ARG, "NULL argument");
+    for (int i = 0; i < g->n; ++i) {
+        frt_status st = frt_stream_configure(g->st[i], cfg);
+        if (st != FRT_OK) return st;
+    }
+    return FRT_OK;
+}
+
+frt_stream_t* frt_steps_stream(const frt_steps_t* g, int step) {
+    if (!g || step < 0 || step >= g->n) return nullptr;
+    return g->st[step];
+}
+
+frt_status frt_steps_tick(frt_steps_t* g, unsigned int active_mask, void* const* q,
+                          void* const* k, const void* const* v, void* const* out) {
+    if (!g || !q || !k || !v || !out) return fail(FRT_ERR_INVALID_ARG, "NULL argument");
+    if (active_mask == 0) return FRT_OK;
+    if (g->n < 32 && (active_mask >> g->n) != 0)
+        return fail(FRT_ERR_INVALID_ARG, "active_mask names a step beyond n_steps");
+    frt_stream_t* streams[kMaxBatchStreams];
+    const void* qs[kMaxBatchStreams];
+    void* outs[kMaxBatchStreams];
+    int n = 0;
+    frt_status st;
+    for (int i = 0; i < g->n; ++i) {
+        if (!((active_mask >> i) & 1u)) continue;
+        if ((st = frt_rope3d_qk(g->st[i], q[i], k[i])) != FRT_OK) return st;
+        if ((st = frt_kv_append_evict(g->st[i], k[i], v[i], nullptr, nullptr)) != FRT_OK) return st;
+        streams[n] = g->st[i];
+        qs[n] = q[i];
+        outs[n] = out[i];
+        ++n;
+    }
+    return frt_chunk_attention_batched(streams, n, qs, outs);
+}
+
+void frt_steps_destroy(frt_steps_t* g) {
+    if (!g) return;
+    for (int i = 0; i < g->n; ++i) frt_stream_destroy(g->st[i]);
+    delete g;
+}
+
+}  // extern "C"

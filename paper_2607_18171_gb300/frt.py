@@ -74,6 +74,12 @@ def lib() -> ctypes.CDLL:
         "frt_selftest_umma_tile": (I, [P, P, P, I, I, I, I, P, P]),
         "frt_selftest_wait_timeout": (I, [P, LL, P]),
         "frt_selftest_umma_pair": (I, [P, P, P, P, P, P]),
+        "frt_steps_create": (P, [I, I, I, I, I, I]),
+        "frt_steps_configure": (I, [P, ctypes.POINTER(Config)]),
+        "frt_steps_stream": (P, [P, I]),
+        "frt_steps_tick": (I, [P, ctypes.c_uint, ctypes.POINTER(P), ctypes.POINTER(P),
+                               ctypes.POINTER(P), ctypes.POINTER(P)]),
+        "frt_steps_destroy": (None, [P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -259,6 +265,67 @@ def chunk_attention_batched(streams, qs, outs) -> None:
     _check(lib().frt_chunk_attention_batched(
         arr(*[s.handle for s in streams]), n, arr(*[q.data_ptr() for q in qs]),
         arr(*[o.data_ptr() for o in outs])))
+
+
+class Steps:
+    """Per-denoising-step caches: n_steps independent streams of one shape advanced by
+    pipeline ticks (frt_steps_* in include/frt.h)."""
+
+    def __init__(self, n_steps: int, heads: int, head_dim: int, grid_h: int, grid_w: int,
+                 frames_per_chunk: int, window_chunks: int, split=None, theta: float = 10000.0,
+                 out_dtype: torch.dtype = torch.float32):
+        L = lib()
+        self._g = L.frt_steps_create(n_steps, heads, head_dim, grid_h * grid_w,
+                                     frames_per_chunk, window_chunks)
+        if not self._g:
+            raise FrtError(1, L.frt_last_error().decode())
+        self.n_steps = n_steps
+        self.n_q = frames_per_chunk * grid_h * grid_w
+        self.heads, self.head_dim, self.out_dtype = heads, head_dim, out_dtype
+        cfg = Config()
+        _check(L.frt_config_default(L.frt_steps_stream(self._g, 0), ctypes.byref(cfg)))
+        cfg.grid_h, cfg.grid_w = grid_h, grid_w
+        if split is not None:
+            cfg.rope_dt, cfg.rope_dh, cfg.rope_dw = (int(x) for x in split)
+        cfg.theta = theta
+        cfg.out_dtype = OUT_BF16 if out_dtype == torch.bfloat16 else OUT_F32
+        cfg.cuda_stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+        _check(L.frt_steps_configure(self._g, ctypes.byref(cfg)))
+
+    def shape(self):
+        return (self.n_q, self.heads, self.head_dim)
+
+    def counter(self, step: int) -> int:
+        return lib().frt_stream_chunk_counter(lib().frt_steps_stream(self._g, step))
+
+    def tick(self, active, q, k, v, out) -> None:
+        """active: iterable of step indices; q/k/v/out: dicts or lists indexed by step."""
+        arr = ctypes.c_void_p * self.n_steps
+        mask = 0
+        ptrs = {n: [None] * self.n_steps for n in ("q", "k", "v", "o")}
+        for i in active:
+            mask |= 1 << i
+            for n, t in (("q", q[i]), ("k", k[i]), ("v", v[i])):
+                _bf16_dev(t, self.shape(), n)
+                ptrs[n][i] = t.data_ptr()
+            ptrs["o"][i] = out[i].data_ptr()
+        _check(lib().frt_steps_tick(self._g, mask, arr(*ptrs["q"]), arr(*ptrs["k"]),
+                                    arr(*ptrs["v"]), arr(*ptrs["o"])))
+
+    def sync(self) -> None:
+        for i in range(self.n_steps):
+            _check(lib().frt_stream_sync(lib().frt_steps_stream(self._g, i)))
+
+    def close(self) -> None:
+        if getattr(self, "_g", None):
+            lib().frt_steps_destroy(self._g)
+            self._g = None
+
+    def __del__(self):  # pragma: no cover - best effort
+        try:
+            self.close()
+        except Exception:
+            pass
 
 
 def selftest_umma_tile(a: torch.Tensor, b: torch.Tensor, b_mn_major: bool, lbo: int = 16384,

@@ -43,6 +43,7 @@ class Workload:
     head_scale: bool = False  # per-head U(0.5, 2) factor on q and k
     ragged_fill: bool = False  # per-stream fill drawn uniform 1..window
     fused_rope: bool = False   # RoPE-Q in the attention prologue
+    steps: int = 1             # denoising steps, each with its own KV cache
 
     @property
     def tokens_per_frame(self) -> int:
@@ -69,6 +70,10 @@ WORKLOADS = {
                            (32, 48, 48), fused_rope=True),
     "multi8": Workload("multi8", 4, 8, 24, 128, 30, 52, 3, 7, 7, (32, 48, 48),
                        ragged_fill=True),
+    # four denoising steps of the 1.3B shape, each with its own cache, advanced in
+    # pipeline ticks (one batched attention launch per tick)
+    "pp4dit1p3b": Workload("pp4dit1p3b", 5, 1, 12, 128, 30, 52, 3, 7, 7, (32, 48, 48),
+                           steps=4),
 }
 
 

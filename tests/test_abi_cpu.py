@@ -114,3 +114,20 @@ def test_product_path_does_not_import_the_oracle():
             if f.endswith(".py"):
                 src = open(os.path.join(dirpath, f)).read()
                 assert not re.search(r"^\s*(import|from)\s+oracle", src, flags=re.M), f
+
+
+def test_step_group_argument_checks(frt):
+    L = frt.lib()
+    assert not L.frt_steps_create(0, 2, 64, 16, 3, 3)
+    assert not L.frt_steps_create(33, 2, 64, 16, 3, 3)
+    assert not L.frt_steps_create(2, 2, 96, 16, 3, 3)      # head_dim unsupported
+    g = L.frt_steps_create(3, 2, 64, 16, 3, 3)
+    assert g
+    assert L.frt_steps_stream(g, 0) and L.frt_steps_stream(g, 2)
+    assert not L.frt_steps_stream(g, 3) and not L.frt_steps_stream(g, -1)
+    # steps are unconfigured: a tick is a state error, an empty tick is a no-op
+    arr = (ctypes.c_void_p * 3)()
+    assert L.frt_steps_tick(g, 0, arr, arr, arr, arr) == 0
+    assert L.frt_steps_tick(g, 0b1000, arr, arr, arr, arr) == 1
+    L.frt_steps_destroy(g)
+    L.frt_steps_destroy(None)
