@@ -153,11 +153,9 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
         }
         mbar_init(smem_u32(&bars->drain[0]), 1);
         mbar_init(smem_u32(&bars->drain[1]), 1);
-        for (int s = 0; s < C::STAGES; ++s) {
-            mbar_init(smem_u32(&bars->kv_full[s]), 1);
+        for (int s = 0; s < C::STAGES; ++s) mbar_init(smem_u32(&bars->kv_full[s]), 1);
         for (int s = 0; s < 4; ++s) mbar_init(smem_u32(&bars->step_done[s]), 1);
         mbar_init(smem_u32(&bars->k0_done), 1);
-        }
         bars->abort_flag = 0;
         fence_mbar_init();
         fence_proxy_async_smem();
