@@ -264,7 +264,7 @@ def run_gpu(args, wl, world, rank, local):
                    "peak": peak_gbs, "unit": "GB/s",
                    "frac": round(app_bytes / (app_ms * 1e-3) / 1e9 / peak_gbs, 4),
                    "frac_of_8tbs": round(app_bytes / (app_ms * 1e-3) / 8e12, 4),
-                   "kernel": "kv_append_kernel (RoPE-K fused)", "launch_ms": round(app_ms, 5),
+                   "kernel": "staged_rows_kernel (KV append, RoPE-K fused)", "launch_ms": round(app_ms, 5),
                    "bytes_per_launch": app_bytes},
         "clocks": clk.summary(),
         "e2e": {"value": round(e2e_value, 2), "unit": UNIT,
