@@ -248,3 +248,54 @@ class OracleStream:
         q_r, k_r = self.rope(q, k)
         slot, evicted = self.append(k_r, v)
         return self.attend(q_r, rows=rows), slot, evicted
+
+
+def linear(x, w) -> np.ndarray:
+    """A linear layer without bias in fp64: ``x`` [tokens, in_features], ``w``
+    [out_features, in_features]; output feature j of a token is the dot product
+    of the token's features with row j of ``w``."""
+    return np.asarray(x, np.float64) @ np.asarray(w, np.float64).T
+
+
+class OracleBlock:
+    """The attention slice of one DiT block over a stream: QKV projection, the
+    chunk step of ``OracleStream`` (RoPE, append/evict, attention), output
+    projection. The paper's video pipelines run their per-chunk attention inside
+    such blocks (section 4.2); it gives no formula for them.
+
+    Readings (the paper is silent): ``w_qkv`` [3d, d] stacks the q, k and v
+    projections in that order (d = heads * head_dim, each output token-major
+    [tokens, heads, head_dim]); no bias and no normalisation; the projection
+    output is rounded to bf16 (q, k, v are bf16 tensors on the whole path) before
+    RoPE, and the attention output is rounded to bf16 before the output
+    projection ``w_o`` [d, d].
+    """
+
+    def __init__(self, w_qkv, w_o, heads: int, head_dim: int, grid_h: int, grid_w: int,
+                 frames_per_chunk: int, window_chunks: int, split, theta: float = 10000.0):
+        self.d = heads * head_dim
+        self.w_qkv = np.asarray(w_qkv, np.float64)
+        self.w_o = np.asarray(w_o, np.float64)
+        assert self.w_qkv.shape == (3 * self.d, self.d) and self.w_o.shape == (self.d, self.d)
+        self.stream = OracleStream(heads, head_dim, grid_h, grid_w, frames_per_chunk,
+                                   window_chunks, split, theta)
+
+    def project_qkv(self, x):
+        """(q, k, v), each [tokens, heads, head_dim], bf16-rounded projections of x."""
+        s = self.stream
+        qkv = bf16_round(linear(x, self.w_qkv))
+        n = qkv.shape[0]
+        return tuple(qkv[:, i * self.d:(i + 1) * self.d].reshape(n, s.heads, s.head_dim)
+                     for i in range(3))
+
+    def step(self, x, rows=None) -> dict:
+        """One frame chunk of hidden states x [Nq, d]. Returns the rotated q and k,
+        v, the attention output o and the block output y (o and y for ``rows``
+        only, if given), and the append's slot / evicted chunk."""
+        q, k, v = self.project_qkv(x)
+        q_r, k_r = self.stream.rope(q, k)
+        slot, evicted = self.stream.append(k_r, v)
+        o = self.stream.attend(q_r, rows=rows)
+        y = linear(bf16_round(o).reshape(o.shape[0], self.d), self.w_o)
+        return {"q_rot": q_r, "k_rot": k_r, "v": v, "o": o, "y": y, "slot": slot,
+                "evicted": evicted}

@@ -15,7 +15,9 @@ generator seeded with SeedSequence([1000*w + s, c]) draws q, k, v (in that
 order) as float32 N(0, 1), optionally multiplied per head by a factor drawn
 U(0.5, 2) once per stream (SeedSequence([1000*w + s, 999999])), then rounded
 to bf16 (round to nearest even). Ragged multi-stream fills are drawn
-uniform on {1..W} from SeedSequence([1000*w, 777777]).
+uniform on {1..W} from SeedSequence([1000*w, 777777]). DiT-block workloads
+draw hidden states x ~ N(0, 1) [Nq, heads*head_dim] per chunk and projection
+weights ~ N(0, 1/d) once per workload (``chunk_x``, ``block_weights``).
 """
 
 from __future__ import annotations
@@ -44,6 +46,7 @@ class Workload:
     ragged_fill: bool = False  # per-stream fill drawn uniform 1..window
     fused_rope: bool = False   # RoPE-Q in the attention prologue
     steps: int = 1             # denoising steps, each with its own KV cache
+    block: bool = False        # DiT-block slice: hidden states x and projection weights
 
     @property
     def tokens_per_frame(self) -> int:
@@ -74,6 +77,11 @@ WORKLOADS = {
     # pipeline ticks (one batched attention launch per tick)
     "pp4dit1p3b": Workload("pp4dit1p3b", 5, 1, 12, 128, 30, 52, 3, 7, 7, (32, 48, 48),
                            steps=4),
+    # the attention slice of a DiT block (QKV projection, RoPE, append, attention,
+    # output projection) around the tiny and the 1.3B shapes
+    "blocktiny": Workload("blocktiny", 6, 1, 2, 64, 4, 4, 3, 3, 4, (16, 24, 24), block=True),
+    "block1p3b": Workload("block1p3b", 7, 1, 12, 128, 30, 52, 3, 7, 7, (32, 48, 48),
+                          block=True),
 }
 
 
@@ -110,6 +118,27 @@ def chunk_qkv(wl: Workload, stream: int, chunk: int):
     """Inputs of ``chunk`` of ``stream`` of workload ``wl``."""
     return random_qkv(wl.n_q, wl.heads, wl.head_dim,
                       [1000 * wl.index + stream, chunk], head_scales(wl, stream))
+
+
+def block_weights(wl: Workload):
+    """(w_qkv [3d, d], w_o [d, d]) bf16 CPU tensors, d = heads * head_dim: entries
+    N(0, 1/d) (so projections of N(0, 1) hidden states are again about N(0, 1)),
+    from PCG64(SeedSequence([1000*w, 555555])), w_qkv drawn first."""
+    d = wl.heads * wl.head_dim
+    rng = np.random.Generator(np.random.PCG64(np.random.SeedSequence([1000 * wl.index, 555555])))
+    sd = np.float32(1.0 / math.sqrt(d))
+    w_qkv = rng.standard_normal((3 * d, d), dtype=np.float32) * sd
+    w_o = rng.standard_normal((d, d), dtype=np.float32) * sd
+    return (torch.from_numpy(w_qkv).to(torch.bfloat16), torch.from_numpy(w_o).to(torch.bfloat16))
+
+
+def chunk_x(wl: Workload, stream: int, chunk: int) -> torch.Tensor:
+    """Hidden states [Nq, d] bf16 of ``chunk``: N(0, 1) from
+    PCG64(SeedSequence([1000*w + stream, chunk, 1]))."""
+    d = wl.heads * wl.head_dim
+    rng = np.random.Generator(np.random.PCG64(
+        np.random.SeedSequence([1000 * wl.index + stream, chunk, 1])))
+    return torch.from_numpy(rng.standard_normal((wl.n_q, d), dtype=np.float32)).to(torch.bfloat16)
 
 
 def as_f64(t: torch.Tensor) -> np.ndarray:
