@@ -168,6 +168,8 @@ def run_gpu(args, wl, world, rank, local):
         return run_gpu_multi(args, wl, world, rank, local, dev, peak_tf, peak_kind)
     if wl.steps > 1:
         return run_gpu_steps(args, wl, world, rank, local, dev, peak_tf, peak_kind)
+    if wl.block:
+        return run_gpu_block(args, wl, world, rank, local, dev, peak_tf, peak_kind)
 
     sid = rank  # each rank streams its own independent video (weak scaling)
     st = frt.Stream(wl.heads, wl.head_dim, wl.grid_h, wl.grid_w, wl.frames, wl.window,
@@ -402,6 +404,104 @@ def run_gpu_steps(args, wl, world, rank, local, dev, peak_tf, peak_kind):
                    "note": "each tick re-rotates the same two input sets in place; timing only"},
         "clocks": clk.summary(),
         "gpu_launches": (2 * wl.steps + 1) * n,
+    }
+
+
+BLOCK_METRIC = ("DiT-block attention-slice TFLOP/s (QKV projection + RoPE + KV append + "
+                "chunk attention + output projection) per frame-chunk at 1 GB300")
+
+
+def run_gpu_block(args, wl, world, rank, local, dev, peak_tf, peak_kind):
+    """One DiT block's attention slice per step (frt_block_step: QKV projection with
+    RoPE and the append in its epilogue, chunk attention, output projection) at steady
+    state (full window), hidden states cycled from a pool larger than L2."""
+    import torch
+    from paper_2607_18171_gb300 import frt, synth
+
+    stream = torch.cuda.current_stream()
+    sid = rank
+    d = wl.heads * wl.head_dim
+    st = frt.Stream(wl.heads, wl.head_dim, wl.grid_h, wl.grid_w, wl.frames, wl.window,
+                    split=wl.split)
+    w_qkv, w_o = (t.to(dev) for t in synth.block_weights(wl))
+    q_buf = torch.empty(wl.n_q, d, dtype=torch.bfloat16, device=dev)
+    o_buf = torch.empty_like(q_buf)
+    ys = [torch.empty(wl.n_q, d, dtype=torch.float32, device=dev) for _ in range(2)]
+    for c in range(wl.window - 1):
+        st.block_step(synth.chunk_x(wl, sid, c).to(dev), w_qkv, w_o, q_buf, o_buf, ys[0])
+    pool = [synth.chunk_x(wl, sid, wl.window - 1 + i).to(dev) for i in range(POOL)]
+    st.sync()
+    attn_flops = wl.attn_flops(wl.window - 1)
+    qkv_flops = 2 * wl.n_q * d * 3 * d
+    out_flops = 2 * wl.n_q * d * d
+    flops = attn_flops + qkv_flops + out_flops
+
+    def step(i):
+        st.block_step(pool[i % POOL], w_qkv, w_o, q_buf, o_buf, ys[i % 2])
+
+    for i in range(args.warmup):
+        step(i)
+    st.sync()
+    n = args.steps
+    ev_a, ev_q, ev_o = (timing_events(n, stream) for _ in range(3))
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        t0.record(stream)
+        for i in range(n):
+            st.set_attention_events(*ev_a[i])
+            st.set_block_events(*ev_q[i], *ev_o[i])
+            step(args.warmup + i)
+        t1.record(stream)
+        torch.cuda.synchronize()
+    st.set_attention_events(None, None)
+    st.set_block_events()
+    st.sync()
+    elapsed = max_over_ranks(t0.elapsed_time(t1), world, dev)
+    attn_ms = statistics.mean(a.elapsed_time(b) for a, b in ev_a)
+    qkv_ms = statistics.mean(a.elapsed_time(b) for a, b in ev_q)
+    out_ms = statistics.mean(a.elapsed_time(b) for a, b in ev_o)
+    st.close()
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    if rank != 0:
+        return None
+
+    def tf(f, ms):
+        return f / (ms * 1e-3) / 1e12
+
+    step_ms = elapsed / n
+    return {
+        "metric": BLOCK_METRIC, "value": round(flops * n * world / (elapsed * 1e-3) / 1e12, 2),
+        "unit": UNIT, "n_gpus": world, "steps": n, "warmup": args.warmup,
+        "ms_per_step": round(step_ms, 4), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) hidden states, N(0,1/d) projection weights)",
+        "config": {"workload": describe(wl) + f", d_model {d}",
+                   "path": "frt_block_step (3 launches: QKV projection with RoPE + append "
+                           "epilogue, chunk attention, output projection)",
+                   "l2": f"{POOL} distinct hidden-state inputs cycled, KV cache "
+                         f"{2 * wl.window * wl.n_q * d * 2 / 1e6:.0f} MB",
+                   "flops_per_step": {"attention": attn_flops, "qkv_projection": qkv_flops,
+                                      "out_projection": out_flops}},
+        "roofline": {"bound": "tensor", "achieved": round(tf(attn_flops, attn_ms), 2),
+                     "peak": peak_tf, "unit": "TFLOP/s",
+                     "frac": round(tf(attn_flops, attn_ms) / peak_tf, 4), "traffic": None,
+                     "kernel": "attn_kernel<128,1,false>", "peak_kind": peak_kind,
+                     "launch_ms": round(attn_ms, 4)},
+        "projections": {
+            "qkv": {"kernel": "gemm_kernel<256> (QKV epilogue)", "launch_ms": round(qkv_ms, 4),
+                    "achieved": round(tf(qkv_flops, qkv_ms), 2),
+                    "frac": round(tf(qkv_flops, qkv_ms) / peak_tf, 4)},
+            "out": {"kernel": "gemm_kernel<256> (plain epilogue, fp32 out)",
+                    "launch_ms": round(out_ms, 4), "achieved": round(tf(out_flops, out_ms), 2),
+                    "frac": round(tf(out_flops, out_ms) / peak_tf, 4)},
+            "unit": "TFLOP/s", "peak": peak_tf},
+        "attention_share_of_step": round(attn_ms / step_ms, 4),
+        "clocks": clk.summary(),
+        "gpu_launches": 3 * n,
     }
 
 

@@ -129,6 +129,40 @@ frt_status frt_chunk_step_host(frt_stream_t* s, const void* q_host,
                                void* out_host, int* slot_out,
                                long long* evicted_out);
 
+/* The attention slice of one DiT block for chunk c: QKV projection -> 3D RoPE
+ * -> KV append/evict -> chunk attention -> output projection (the DiT blocks of
+ * the paper's video pipelines, section 4.2, are where the chunk attention runs).
+ *   x      [Nq, d] bf16, the chunk's hidden states (d = heads * head_dim);
+ *   w_qkv  [3d, d] bf16, row-major (output features x input features): rows
+ *          [0, d) produce q, [d, 2d) k, [2d, 3d) v, each token-major
+ *          [Nq, heads, head_dim];
+ *   w_o    [d, d] bf16, same convention;
+ *   q_buf  [Nq, d] bf16 caller-owned work buffer: receives the rotated q;
+ *   o_buf  [Nq, d] bf16 caller-owned work buffer: receives the attention output;
+ *   y      [Nq, d] in the stream's out dtype (fp32 or bf16): o_buf . w_o^T.
+ * Three launches on the stream's CUDA stream: the QKV projection (its epilogue
+ * rounds q/k/v to bf16, rotates q and k, writes q to q_buf and k, v straight
+ * into ring slot c mod W), the attention (bf16 output into o_buf), the output
+ * projection. Projections accumulate in fp32 on the tensor cores. The chunk
+ * counter advances as for frt_kv_append_evict; slot_out / evicted_out (may be
+ * NULL) as there. Requires d % 128 == 0. Allowed at the start of a chunk. */
+frt_status frt_block_step(frt_stream_t* s, const void* x, const void* w_qkv,
+                          const void* w_o, void* q_buf, void* o_buf, void* y,
+                          int* slot_out, long long* evicted_out);
+
+/* Plain projection C = A . B^T on the tensor cores (the kernel the block step
+ * uses, without its QKV epilogue): A [M, K] bf16 row-major, B [N, K] bf16
+ * row-major, C [M, ldc] row-major fp32 (c_dtype FRT_OUT_F32) or bf16
+ * (FRT_OUT_BF16), rows/columns past M/N untouched; fp32 accumulation, bf16
+ * output rounded to nearest even. K % 8 == 0, ldc >= N, ldc * element size a
+ * multiple of 16 bytes, pointers 16-byte aligned. `status` (may be NULL) is a
+ * device-visible int[4] that a device-side bounded wait that gave up fills with
+ * FRT_ERR_TIMEOUT (it must start zeroed). Enqueued on cuda_stream
+ * (cudaStream_t; NULL = legacy default stream). */
+frt_status frt_gemm_bf16(const void* a, const void* b, void* c, int M, int N,
+                         int K, int ldc, int c_dtype, void* status,
+                         void* cuda_stream);
+
 /* Operation 3 for n independent streams in one launch (ragged KV lengths):
  * each streams[i] must have just appended (as for frt_chunk_attention); q[i]
  * and out[i] are that stream's rotated queries and output. All streams must
@@ -216,6 +250,13 @@ frt_status frt_stream_set_attention_events(frt_stream_t* s, void* start_event,
 /* Instrumentation: the same for every KV append kernel launch of s
  * (frt_kv_append_evict and the append inside frt_chunk_step). */
 frt_status frt_stream_set_append_events(frt_stream_t* s, void* start_event, void* stop_event);
+
+/* Instrumentation for frt_block_step: events recorded immediately before and
+ * after its QKV projection (qkv_*) and its output projection (out_*) launches;
+ * the attention launch uses the attention events. NULLs turn it off. */
+frt_status frt_stream_set_block_events(frt_stream_t* s, void* qkv_start,
+                                       void* qkv_stop, void* out_start,
+                                       void* out_stop);
 
 /* Index of the next chunk to be appended (chunks appended so far). */
 long long frt_stream_chunk_counter(const frt_stream_t* s);

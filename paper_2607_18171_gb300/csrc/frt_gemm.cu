@@ -1,0 +1,330 @@
+// frt_gemm.cu — C = A · B^T on the sm_103a tensor cores: bf16 operands (both K-major),
+// fp32 accumulation in TMEM, for the linear projections around the chunk attention of a
+// DiT block (QKV projection in front of it, output projection after it).
+//
+// Persistent kernel, one CTA per SM, 192 threads:
+//   warp 0      TMA producer: A (128 x 64) and B (BN x 64) k-blocks, 128-byte swizzle,
+//               through a kStages-deep shared-memory ring;
+//   warp 1      TMEM allocator + single-thread tcgen05.mma issuer (M = 128, N = BN, K = 16
+//               per instruction, four per k-block);
+//   warps 2-5   epilogue: one thread per accumulator row (TMEM lane), 32 columns per
+//               tcgen05.ld.
+// The accumulator is double-buffered in TMEM (2 x BN columns), so the epilogue of tile i
+// runs while the tensor pipe computes tile i + 1.
+//
+// Epilogues:
+//   plain  C row-major, fp32 or bf16 (round to nearest even), rows >= M and columns >= N
+//          are not stored;
+//   qkv    the QKV projection of a frame chunk: columns [0, d) are q, [d, 2d) k, [2d, 3d)
+//          v (d = heads * head_dim). Values are rounded to bf16 first, then q and k are
+//          rotated with the same 3D RoPE routine as every other kernel (so the result is
+//          bit-identical to a plain bf16 projection followed by the RoPE kernel); q goes
+//          to its buffer, k and v straight into the chunk's ring slot of the KV cache.
+//
+// Every wait is bounded: a role that gives up records FRT_ERR_TIMEOUT in the status
+// block, raises the CTA's abort flag, drains its in-flight copies / MMAs and the CTA
+// frees TMEM before exiting.
+#include "frt_internal.h"
+#include "frt_ptx.cuh"
+
+namespace frt {
+
+namespace {
+
+constexpr int kThreads = 192;
+constexpr int kBM = 128;
+constexpr int kBK = 64;          // one 128-byte swizzle atom of bf16
+constexpr int kStages = 4;
+constexpr int kTimeoutCode = 6;  // FRT_ERR_TIMEOUT
+
+template <int BN>
+struct GCfg {
+    static constexpr int A_BYTES = kBM * kBK * 2;
+    static constexpr int B_BYTES = BN * kBK * 2;
+    static constexpr int STAGE = A_BYTES + B_BYTES;
+    static constexpr int SMEM = kStages * STAGE + 1024;   // + alignment slack
+    static constexpr uint32_t IDESC = idesc_bf16_f32(kBM, BN, false);
+    static constexpr uint32_t TMEM_COLS = 2 * BN;
+};
+
+struct GBars {
+    uint64_t full[kStages];
+    uint64_t empty[kStages];
+    uint64_t acc_full[2];
+    uint64_t acc_empty[2];
+    uint64_t drain;
+    uint32_t tmem_base;
+    int abort_flag;
+};
+
+__device__ __forceinline__ void report(DeviceStatus* st, volatile int* abort, int role, int where) {
+    *abort = 1;
+    if (st != nullptr) {
+        volatile DeviceStatus* s = st;
+        if (s->code == 0) {
+            s->block = blockIdx.x;
+            s->role = 200 + role;
+            s->where = where;
+            __threadfence_system();
+            s->code = kTimeoutCode;
+        }
+    }
+}
+
+template <int BN>
+__global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant__ GemmParams p) {
+    using C = GCfg<BN>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~uintptr_t(1023));
+    __shared__ GBars bars;
+    __shared__ float2 s_t[kMaxTEntries];
+    const uint32_t sbase = smem_u32(smem);
+    volatile int* abort = &bars.abort_flag;
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int n_tiles = p.tiles_m * p.tiles_n;
+    const int nk = (p.K + kBK - 1) / kBK;
+    const uint64_t lim = p.wait_limit_ns;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(smem_u32(&bars.full[s]), 1);
+            mbar_init(smem_u32(&bars.empty[s]), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_u32(&bars.acc_full[b]), 1);
+            mbar_init(smem_u32(&bars.acc_empty[b]), 128);
+        }
+        mbar_init(smem_u32(&bars.drain), 1);
+        bars.abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (p.epi == kEpiQkv && p.rope)
+        for (int i = threadIdx.x; i < kMaxTEntries; i += kThreads) s_t[i] = p.ra.t_tab[i];
+    if (warp == 1) {
+        tmem_alloc(smem_u32(&bars.tmem_base), C::TMEM_COLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = bars.tmem_base;
+
+    if (warp == 0) {
+        // ==================================== TMA producer ===================================
+        if (lane == 0) {
+            tma_prefetch_map(&p.a_map);
+            tma_prefetch_map(&p.b_map);
+            int it = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+                const int tm = t % p.tiles_m;
+                const int tn = t / p.tiles_m;
+                for (int kb = 0; kb < nk; ++kb) {
+                    const int s = it % kStages;
+                    // slot s was last filled by load it - kStages; the MMA that read it
+                    // commits empty[s] once per use
+                    if (it >= kStages &&
+                        !mbar_wait(smem_u32(&bars.empty[s]), ((it / kStages) - 1) & 1, lim, abort)) {
+                        report(p.status, abort, 0, it);
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t fb = smem_u32(&bars.full[s]);
+                    mbar_arrive_expect_tx(fb, C::STAGE);
+                    const uint32_t dst = sbase + s * C::STAGE;
+                    tma_load_2d(dst, &p.a_map, fb, kb * kBK, tm * kBM);
+                    tma_load_2d(dst + C::A_BYTES, &p.b_map, fb, kb * kBK, tn * BN);
+                    ++it;
+                }
+            }
+            // drain: every issued load lands before the CTA may exit
+            for (int i = (it > kStages ? it - kStages : 0); i < it; ++i)
+                mbar_wait_drain(smem_u32(&bars.full[i % kStages]), (i / kStages) & 1, lim);
+        }
+    } else if (warp == 1) {
+        // ============================ MMA issuer (one thread) ===============================
+        if (lane == 0) {
+            // descriptors are linear in the 16-byte start address: a K step of 16 bf16
+            // inside the 128-byte swizzle atom adds 32 bytes (2 units)
+            const uint64_t da0 = sdesc_sw128(sbase, 16, 1024);
+            const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, 16, 1024);
+            int it = 0;
+            int tl = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++tl) {
+                const int b = tl & 1;
+                if (tl >= 2 &&
+                    !mbar_wait(smem_u32(&bars.acc_empty[b]), ((tl >> 1) - 1) & 1, lim, abort)) {
+                    report(p.status, abort, 1, -1 - tl);
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t d = tmem + uint32_t(b * BN);
+                for (int kb = 0; kb < nk; ++kb, ++it) {
+                    const int s = it % kStages;
+                    if (!mbar_wait(smem_u32(&bars.full[s]), (it / kStages) & 1, lim, abort)) {
+                        report(p.status, abort, 1, it);
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint64_t so = uint64_t((s * C::STAGE) >> 4);
+#pragma unroll
+                    for (int k = 0; k < kBK / 16; ++k)
+                        umma_ss(d, da0 + so + uint64_t(2 * k), db0 + so + uint64_t(2 * k), C::IDESC,
+                                (kb > 0 || k > 0) ? 1u : 0u);
+                    umma_commit(smem_u32(&bars.empty[s]));
+                }
+                if (ok) umma_commit(smem_u32(&bars.acc_full[b]));
+            }
+            // drain: all issued MMAs complete before TMEM is released
+            umma_commit(smem_u32(&bars.drain));
+            mbar_wait_drain(smem_u32(&bars.drain), 0, lim);
+        }
+    } else {
+        // ====================================== epilogue =====================================
+        const int sub = warp & 3;                      // TMEM lane quarter of this warp
+        const int row = sub * 32 + lane;
+        const uint32_t lane_off = uint32_t(sub * 32) << 16;
+        int tl = 0;
+        for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++tl) {
+            const int b = tl & 1;
+            const int tm = t % p.tiles_m;
+            const int tn = t / p.tiles_m;
+            const bool got = mbar_wait(smem_u32(&bars.acc_full[b]), (tl >> 1) & 1, lim, abort);
+            if (!__all_sync(0xffffffffu, got)) {
+                if (!got) report(p.status, abort, 2, tl);
+                break;
+            }
+            tc_fence_after();
+            const int grow = tm * kBM + row;
+            const bool live = grow < p.M;
+            const int n0 = tn * BN;
+            if (p.epi == kEpiQkv) {
+                const int which = n0 / p.d;                 // 0 q, 1 k, 2 v
+                const int cbase = n0 - which * p.d;
+                uint16_t* dst = which == 0 ? p.q_out : (which == 1 ? p.k_out : p.v_out);
+                const bool rot = p.rope && which < 2;
+                int f = 0, rr = 0, col = 0;
+                if (rot) {
+                    f = grow / p.ra.tpf;
+                    const int rem = grow - f * p.ra.tpf;
+                    rr = rem / p.ra.gw;
+                    col = rem - rr * p.ra.gw;
+                }
+#pragma unroll 1
+                for (int c = 0; c < BN / 32; ++c) {
+                    uint32_t r[32];
+                    tmem_ld32(tmem + lane_off + uint32_t(b * BN + c * 32), r);
+                    tmem_ld_wait();
+                    if (live) {
+                    const int cc = cbase + c * 32;
+                    uint32_t w[16];
+#pragma unroll
+                    for (int i = 0; i < 16; ++i)
+                        w[i] = pack_bf16x2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
+                    if (rot) {
+                        const int pi0 = (cc & (p.head_dim - 1)) >> 1;
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) {
+                            const float2 cs = rope_cs(p.ra, s_t, pi0 + i, f, rr, col);
+                            w[i] = rope_pair(w[i], cs.x, cs.y);
+                        }
+                    }
+                    uint4* o = reinterpret_cast<uint4*>(dst + size_t(grow) * p.d + cc);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        o[i] = make_uint4(w[4 * i], w[4 * i + 1], w[4 * i + 2], w[4 * i + 3]);
+                    }
+                    __syncwarp();
+                }
+            } else {
+#pragma unroll 1
+                for (int c = 0; c < BN / 32; ++c) {
+                    uint32_t r[32];
+                    tmem_ld32(tmem + lane_off + uint32_t(b * BN + c * 32), r);
+                    tmem_ld_wait();
+                    const int c0 = n0 + c * 32;
+                    if (live && c0 < p.N) {
+                    const size_t off = size_t(grow) * p.ldc + c0;
+                    if (c0 + 32 <= p.N) {
+                        if (p.c_bf16) {
+                            uint4* o = reinterpret_cast<uint4*>(static_cast<uint16_t*>(p.c) + off);
+#pragma unroll
+                            for (int i = 0; i < 4; ++i)
+                                o[i] = make_uint4(
+                                    pack_bf16x2(__uint_as_float(r[8 * i + 0]), __uint_as_float(r[8 * i + 1])),
+                                    pack_bf16x2(__uint_as_float(r[8 * i + 2]), __uint_as_float(r[8 * i + 3])),
+                                    pack_bf16x2(__uint_as_float(r[8 * i + 4]), __uint_as_float(r[8 * i + 5])),
+                                    pack_bf16x2(__uint_as_float(r[8 * i + 6]), __uint_as_float(r[8 * i + 7])));
+                        } else {
+                            uint4* o = reinterpret_cast<uint4*>(static_cast<float*>(p.c) + off);
+#pragma unroll
+                            for (int i = 0; i < 8; ++i)
+                                o[i] = make_uint4(r[4 * i], r[4 * i + 1], r[4 * i + 2], r[4 * i + 3]);
+                        }
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) {
+                            if (c0 + i >= p.N) continue;
+                            const float v = __uint_as_float(r[i]);
+                            if (p.c_bf16) {
+                                static_cast<uint16_t*>(p.c)[off + i] =
+                                    uint16_t(pack_bf16x2(v, 0.0f) & 0xFFFFu);
+                            } else {
+                                static_cast<float*>(p.c)[off + i] = v;
+                            }
+                        }
+                    }
+                    }
+                    __syncwarp();
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(smem_u32(&bars.acc_empty[b]));
+        }
+    }
+    __syncwarp();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc(tmem, C::TMEM_COLS);
+}
+
+template <int BN>
+cudaError_t launch(const GemmParams& p, cudaStream_t st) {
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(gemm_kernel<BN>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             GCfg<BN>::SMEM);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    const int n_tiles = p.tiles_m * p.tiles_n;
+    const int grid = n_tiles < num_sms() ? n_tiles : num_sms();
+    gemm_kernel<BN><<<grid, kThreads, GCfg<BN>::SMEM, st>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+int gemm_block_n(int N, int epi, int d) {
+    // BN = 256 unless the QKV epilogue needs 128-column tiles (d not a multiple of 256)
+    // or N is small enough that 128-column tiles fill more SMs
+    if (epi == kEpiQkv) return (d % 256 == 0) ? 256 : 128;
+    return (N > 128) ? 256 : 128;
+}
+
+cudaError_t launch_gemm(GemmParams p, cudaStream_t st) {
+    if (p.M <= 0 || p.N <= 0 || p.K <= 0) return cudaSuccess;
+    const int bn = gemm_block_n(p.N, p.epi, p.d);
+    p.tiles_m = (p.M + kBM - 1) / kBM;
+    p.tiles_n = (p.N + bn - 1) / bn;
+    return bn == 256 ? launch<256>(p, st) : launch<128>(p, st);
+}
+
+}  // namespace frt

@@ -72,6 +72,23 @@ frt_status make_map(CUtensorMap* map, const void* base, int head_dim, int heads,
     return FRT_OK;
 }
 
+// 2D map over a row-major [rows, K] bf16 matrix; box = 64 columns x box_rows rows,
+// 128-byte swizzle; rows and columns past the extent read as zero.
+frt_status make_map_2d(CUtensorMap* map, const void* base, long long K, long long rows,
+                       int box_rows) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return fail(FRT_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+    cuuint64_t dims[2] = {cuuint64_t(K), cuuint64_t(rows)};
+    cuuint64_t strides[1] = {cuuint64_t(K) * 2};
+    cuuint32_t box[2] = {64, cuuint32_t(box_rows)};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims,
+                    strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(FRT_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", int(r));
+    return FRT_OK;
+}
+
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 enum Phase { kStart = 0, kRoped = 1, kAppended = 2 };
@@ -112,6 +129,10 @@ struct frt_stream {
     cudaEvent_t attn_stop = nullptr;
     cudaEvent_t app_start = nullptr;
     cudaEvent_t app_stop = nullptr;
+    cudaEvent_t qkv_start = nullptr;   // frt_block_step projections
+    cudaEvent_t qkv_stop = nullptr;
+    cudaEvent_t proj_start = nullptr;
+    cudaEvent_t proj_stop = nullptr;
     // split-KV scratch: partial O / (max, sum) per (query group, split), one counter per
     // query group (zero between launches)
     float* part_o = nullptr;
@@ -212,7 +233,9 @@ int log2_exact(int x) {
     return l;
 }
 
-frt_status attention_single(frt_stream_t* s, const void* q, void* out, bool rope_q) {
+// out_bf16: 1 / 0 force the output dtype, -1 takes the stream's configured one.
+frt_status attention_single(frt_stream_t* s, const void* q, void* out, bool rope_q,
+                            int out_bf16 = -1) {
     AttnParams<1> p;
     std::memset(&p, 0, sizeof(p));
     const long long n_valid = std::min<long long>(s->counter, s->window);
@@ -236,7 +259,7 @@ frt_status attention_single(frt_stream_t* s, const void* q, void* out, bool rope
     p.n_streams = 1;
     p.heads = s->heads;
     p.total_items = int(groups * p.n_split);
-    p.out_bf16 = s->cfg.out_dtype == FRT_OUT_BF16;
+    p.out_bf16 = out_bf16 >= 0 ? out_bf16 : (s->cfg.out_dtype == FRT_OUT_BF16);
     p.scale_log2 = float(double(s->scale) * 1.4426950408889634);
     p.wait_limit_ns = s->wait_limit_ns;
     p.status = s->status_dev;
@@ -547,6 +570,112 @@ frt_status frt_chunk_step(frt_stream_t* s, const void* q, const void* k, const v
     return attention_single(s, q, out, true);
 }
 
+frt_status frt_block_step(frt_stream_t* s, const void* x, const void* w_qkv, const void* w_o,
+                          void* q_buf, void* o_buf, void* y, int* slot_out,
+                          long long* evicted_out) {
+    frt_status st = require_configured(s);
+    if (st != FRT_OK) return st;
+    if (!x || !w_qkv || !w_o || !q_buf || !o_buf || !y || !aligned16(x) || !aligned16(w_qkv) ||
+        !aligned16(w_o) || !aligned16(q_buf) || !aligned16(o_buf) || !aligned16(y))
+        return fail(FRT_ERR_INVALID_ARG,
+                    "x, w_qkv, w_o, q_buf, o_buf, y must be non-NULL and 16-byte aligned");
+    if (s->phase == kRoped) return fail(FRT_ERR_STATE, "a separate rope is pending");
+    const int d = s->heads * s->head_dim;
+    if (d % 128 != 0)
+        return fail(FRT_ERR_UNSUPPORTED, "heads * head_dim must be a multiple of 128");
+    int slot;
+    long long evicted;
+    frt_window_index(s->counter, s->window, &slot, &evicted, nullptr);
+    const size_t off = size_t(slot) * s->chunk_elems;
+
+    // 1. QKV projection; its epilogue rotates q, k and writes k, v into the ring slot
+    GemmParams g;
+    std::memset(&g, 0, sizeof(g));
+    const int bn = gemm_block_n(3 * d, kEpiQkv, d);
+    if ((st = make_map_2d(&g.a_map, x, d, s->n_q, 128)) != FRT_OK) return st;
+    if ((st = make_map_2d(&g.b_map, w_qkv, d, 3LL * d, bn)) != FRT_OK) return st;
+    g.M = s->n_q;
+    g.N = 3 * d;
+    g.K = d;
+    g.epi = kEpiQkv;
+    g.d = d;
+    g.head_dim = s->head_dim;
+    g.q_out = static_cast<uint16_t*>(q_buf);
+    g.k_out = static_cast<uint16_t*>(s->cache_k) + off;
+    g.v_out = static_cast<uint16_t*>(s->cache_v) + off;
+    g.rope = 1;
+    fill_rope(s, s->counter, g.ra);
+    g.wait_limit_ns = s->wait_limit_ns;
+    g.status = s->status_dev;
+    cudaError_t e = cudaSuccess;
+    if (s->qkv_start) e = cudaEventRecord(s->qkv_start, s->cs);
+    if (e == cudaSuccess) e = launch_gemm(g, s->cs);
+    if (e == cudaSuccess && s->qkv_stop) e = cudaEventRecord(s->qkv_stop, s->cs);
+    if (e != cudaSuccess) return cuda_fail(e, "QKV projection launch");
+    s->counter += 1;
+    s->phase = kAppended;
+    s->last_q = q_buf;
+    s->last_k = nullptr;
+    s->last_v = nullptr;
+    if (slot_out) *slot_out = slot;
+    if (evicted_out) *evicted_out = evicted;
+
+    // 2. attention of the chunk (q already rotated), bf16 output for the projection
+    if ((st = attention_single(s, q_buf, o_buf, false, 1)) != FRT_OK) return st;
+
+    // 3. output projection
+    GemmParams h;
+    std::memset(&h, 0, sizeof(h));
+    const int bn2 = gemm_block_n(d, kEpiPlain, 0);
+    if ((st = make_map_2d(&h.a_map, o_buf, d, s->n_q, 128)) != FRT_OK) return st;
+    if ((st = make_map_2d(&h.b_map, w_o, d, d, bn2)) != FRT_OK) return st;
+    h.M = s->n_q;
+    h.N = d;
+    h.K = d;
+    h.epi = kEpiPlain;
+    h.c = y;
+    h.ldc = d;
+    h.c_bf16 = s->cfg.out_dtype == FRT_OUT_BF16;
+    h.wait_limit_ns = s->wait_limit_ns;
+    h.status = s->status_dev;
+    if (s->proj_start) e = cudaEventRecord(s->proj_start, s->cs);
+    if (e == cudaSuccess) e = launch_gemm(h, s->cs);
+    if (e == cudaSuccess && s->proj_stop) e = cudaEventRecord(s->proj_stop, s->cs);
+    if (e != cudaSuccess) return cuda_fail(e, "output projection launch");
+    return FRT_OK;
+}
+
+frt_status frt_gemm_bf16(const void* a, const void* b, void* c, int M, int N, int K, int ldc,
+                         int c_dtype, void* status, void* cuda_stream) {
+    if (!a || !b || !c || !aligned16(a) || !aligned16(b) || !aligned16(c) ||
+        (status && (reinterpret_cast<uintptr_t>(status) & 3u)))
+        return fail(FRT_ERR_INVALID_ARG, "a, b, c must be non-NULL and 16-byte aligned");
+    if (M < 1 || N < 1 || K < 1 || K % 8 != 0 || ldc < N)
+        return fail(FRT_ERR_INVALID_ARG, "need M, N, K >= 1, K %% 8 == 0 and ldc >= N");
+    if (c_dtype != FRT_OUT_F32 && c_dtype != FRT_OUT_BF16)
+        return fail(FRT_ERR_INVALID_ARG, "unknown c_dtype");
+    const int esz = c_dtype == FRT_OUT_BF16 ? 2 : 4;
+    if ((long long)ldc * esz % 16 != 0)
+        return fail(FRT_ERR_INVALID_ARG, "ldc * element size must be a multiple of 16 bytes");
+    GemmParams g;
+    std::memset(&g, 0, sizeof(g));
+    frt_status st;
+    if ((st = make_map_2d(&g.a_map, a, K, M, 128)) != FRT_OK) return st;
+    if ((st = make_map_2d(&g.b_map, b, K, N, gemm_block_n(N, kEpiPlain, 0))) != FRT_OK) return st;
+    g.M = M;
+    g.N = N;
+    g.K = K;
+    g.epi = kEpiPlain;
+    g.c = c;
+    g.ldc = ldc;
+    g.c_bf16 = c_dtype == FRT_OUT_BF16;
+    g.wait_limit_ns = kDefaultWaitLimitNs;
+    g.status = static_cast<DeviceStatus*>(status);
+    cudaError_t e = launch_gemm(g, static_cast<cudaStream_t>(cuda_stream));
+    if (e != cudaSuccess) return cuda_fail(e, "projection launch");
+    return FRT_OK;
+}
+
 frt_status frt_chunk_step_host(frt_stream_t* s, const void* q_host, const void* k_host,
                                const void* v_host, void* out_host, int* slot_out,
                                long long* evicted_out) {
@@ -740,6 +869,16 @@ void frt_stream_destroy(frt_stream_t* s) {
     if (s->configured) cudaStreamSynchronize(s->cs);
     free_device(s);
     delete s;
+}
+
+frt_status frt_stream_set_block_events(frt_stream_t* s, void* qkv_start, void* qkv_stop,
+                                       void* out_start, void* out_stop) {
+    if (s == nullptr) return fail(FRT_ERR_INVALID_ARG, "NULL stream handle");
+    s->qkv_start = static_cast<cudaEvent_t>(qkv_start);
+    s->qkv_stop = static_cast<cudaEvent_t>(qkv_stop);
+    s->proj_start = static_cast<cudaEvent_t>(out_start);
+    s->proj_stop = static_cast<cudaEvent_t>(out_stop);
+    return FRT_OK;
 }
 
 long long frt_stream_chunk_counter(const frt_stream_t* s) { return s ? s->counter : -1; }

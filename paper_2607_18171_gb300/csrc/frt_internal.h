@@ -126,7 +126,38 @@ struct RopeParams {
     RopeArgs ra;
 };
 
+// ----------------------------------------------------------------------------------------
+// Linear projections (C = A . B^T, bf16 operands, fp32 accumulation)
+// ----------------------------------------------------------------------------------------
+constexpr int kEpiPlain = 0;   // C row-major, fp32 or bf16
+constexpr int kEpiQkv = 1;     // DiT-block QKV projection: q -> q_out, k/v -> cache slot
+
+struct GemmParams {
+    CUtensorMap a_map;      // 2D (K, M) bf16, box (64, 128), 128-byte swizzle
+    CUtensorMap b_map;      // 2D (K, N) bf16, box (64, BN), 128-byte swizzle
+    int M, N, K;
+    int tiles_m, tiles_n;   // filled in by launch_gemm
+    int epi;
+    // plain epilogue
+    void* c;
+    int ldc;                // elements
+    int c_bf16;
+    // QKV epilogue: N = 3 d, d = heads * head_dim, each destination [M, d] bf16
+    int d;
+    int head_dim;
+    uint16_t* q_out;
+    uint16_t* k_out;
+    uint16_t* v_out;
+    int rope;               // rotate q and k (3D RoPE at the chunk's positions)
+    unsigned long long wait_limit_ns;
+    DeviceStatus* status;
+    RopeArgs ra;
+};
+
 // Kernel launchers (defined in the .cu files).
+cudaError_t launch_gemm(GemmParams p, cudaStream_t st);
+// Column tile width the GEMM uses for this problem (the B tensor map's box height).
+int gemm_block_n(int N, int epi, int d);
 cudaError_t launch_rope_qk(const RopeParams& p, cudaStream_t st);
 cudaError_t launch_kv_append(const AppendParams& p, cudaStream_t st);
 cudaError_t launch_attention_single(const AttnParams<1>& p, int head_dim, bool rope_q,

@@ -66,6 +66,9 @@ def lib() -> ctypes.CDLL:
         "frt_stream_set_attention_events": (I, [P, P, P]),
         "frt_stream_set_append_events": (I, [P, P, P]),
         "frt_chunk_attention_noalloc": (I, [P, P, P, P, I, I, I, I, D, I, P, P]),
+        "frt_block_step": (I, [P, P, P, P, P, P, P, ctypes.POINTER(I), ctypes.POINTER(LL)]),
+        "frt_gemm_bf16": (I, [P, P, P, I, I, I, I, I, P, P]),
+        "frt_stream_set_block_events": (I, [P, P, P, P, P]),
         "frt_window_index": (I, [LL, I, ctypes.POINTER(I), ctypes.POINTER(LL),
                                  ctypes.POINTER(I)]),
         "frt_status_string": (ctypes.c_char_p, [I]),
@@ -206,6 +209,30 @@ class Stream:
                                          _ptr(out_host), ctypes.byref(slot), ctypes.byref(ev)))
         return slot.value, ev.value
 
+    def block_step(self, x, w_qkv, w_o, q_buf, o_buf, y):
+        """DiT-block attention slice of the next chunk: x [Nq, d] -> y [Nq, d]
+        (d = heads * head_dim); q_buf / o_buf are [Nq, d] bf16 work buffers."""
+        n_q = self.shape()[0]
+        d = self.heads * self.head_dim
+        _bf16_dev(x, (n_q, d), "x")
+        _bf16_dev(w_qkv, (3 * d, d), "w_qkv")
+        _bf16_dev(w_o, (d, d), "w_o")
+        _bf16_dev(q_buf, (n_q, d), "q_buf")
+        _bf16_dev(o_buf, (n_q, d), "o_buf")
+        if y.dtype != self.out_dtype or not y.is_cuda or not y.is_contiguous() or \
+                tuple(y.shape) != (n_q, d):
+            raise ValueError("y must be a contiguous [Nq, d] CUDA tensor of the stream's out dtype")
+        slot, ev = ctypes.c_int(), ctypes.c_longlong()
+        _check(lib().frt_block_step(self._h, _ptr(x), _ptr(w_qkv), _ptr(w_o), _ptr(q_buf),
+                                    _ptr(o_buf), _ptr(y), ctypes.byref(slot), ctypes.byref(ev)))
+        return slot.value, ev.value
+
+    def set_block_events(self, qkv_start=None, qkv_stop=None, out_start=None, out_stop=None):
+        """Record events around the two projection launches of block_step."""
+        ev = [None if e is None else ctypes.c_void_p(e.cuda_event)
+              for e in (qkv_start, qkv_stop, out_start, out_stop)]
+        _check(lib().frt_stream_set_block_events(self._h, *ev))
+
     def sync(self) -> None:
         _check(lib().frt_stream_sync(self._h))
 
@@ -326,6 +353,30 @@ class Steps:
             self.close()
         except Exception:
             pass
+
+
+def gemm_bf16(a: torch.Tensor, b: torch.Tensor, c: torch.Tensor,
+              status: torch.Tensor | None = None) -> None:
+    """c[:M, :N] = a @ b.T on the tensor cores (a [M, K], b [N, K] bf16; c fp32 or bf16,
+    row stride c.stride(0)); enqueued on torch's current CUDA stream."""
+    for t, n in ((a, "a"), (b, "b")):
+        if t.dtype != torch.bfloat16 or not t.is_cuda or not t.is_contiguous() or t.dim() != 2:
+            raise ValueError(f"{n} must be a contiguous 2D bf16 CUDA tensor")
+    M, K = a.shape
+    N = b.shape[0]
+    if b.shape[1] != K:
+        raise ValueError("a and b disagree on K")
+    if c.dim() != 2 or c.stride(1) != 1 or not c.is_cuda or c.shape[0] < M or c.shape[1] < N:
+        raise ValueError("c must be a row-major CUDA matrix of at least [M, N]")
+    if c.dtype == torch.float32:
+        cd = OUT_F32
+    elif c.dtype == torch.bfloat16:
+        cd = OUT_BF16
+    else:
+        raise ValueError("c must be float32 or bfloat16")
+    _check(lib().frt_gemm_bf16(_ptr(a), _ptr(b), _ptr(c), M, N, K, c.stride(0), cd,
+                               _ptr(status),
+                               ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)))
 
 
 def selftest_umma_tile(a: torch.Tensor, b: torch.Tensor, b_mn_major: bool, lbo: int = 16384,
