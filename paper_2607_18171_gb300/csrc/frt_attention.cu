@@ -187,8 +187,10 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             // Load L reuses the ring slot of load L - STAGES. Slots are released per KV
             // step: step j reads V_j and K_{j+1} (loads 2j+1, 2j+2) and its single release
             // commit arrives on step_done[j % 4]; K_0 (load 0) is released by k0_done.
-            // Step j+4 needs loads the producer has not issued while it waits for step
-            // j, so the parity of step_done[j % 4] is never ambiguous.
+            // The MMA thread issues that commit early in step j+1 (inside PV_0(j+1), which
+            // needs only loads up to 2j+4, whose slots step j-1 released). Step j+4's
+            // commit needs loads the producer has not issued while it waits for step j,
+            // so the parity of step_done[j % 4] is never ambiguous.
             int L = 0;
             for (; L < n_loads; ++L) {
                 const int stage = L % C::STAGES;
@@ -297,7 +299,12 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 // V_j has been waited for; K_{j+1} is waited for inside PV_0(j);
                 // V_{j+1} inside the last group of this step.
                 if (!(ok = wait_p(0, j))) break;
-                issue_o(0, sv, j > 0, [&](int k) { if (k == 0 && more) ok = wait_load(2 * j + 2); });
+                // the release of step j-1 rides in the shadow of PV_0(j)'s second MMA
+                // instead of idling the tensor pipe at the end of step j-1
+                issue_o(0, sv, j > 0, [&](int k) {
+                    if (k == 0 && more) ok = wait_load(2 * j + 2);
+                    if (k == 1 && j > 0) umma_commit(smem_u32(&bars->step_done[(j - 1) & 3]));
+                });
                 if (!ok) break;
                 if (ng == 2) {
                     if (more) issue_s(0, sk, nop);
@@ -306,11 +313,9 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                     issue_o(1, sv, j > 0, nop);
                     if (more) issue_s(1, sk, [&](int k) { if (k == 0) ok = wait_load(2 * j + 3); });
                     else umma_commit(smem_u32(&bars->o_done[1]));
-                    if (more) umma_commit(smem_u32(&bars->step_done[j & 3]));
                 } else {
                     if (more) issue_s(0, sk, [&](int k) { if (k == 0) ok = wait_load(2 * j + 3); });
                     else umma_commit(smem_u32(&bars->o_done[0]));
-                    if (more) umma_commit(smem_u32(&bars->step_done[j & 3]));
                 }
                 sv = (sv + 2 >= C::STAGES) ? sv + 2 - C::STAGES : sv + 2;
                 sk = (sk + 2 >= C::STAGES) ? sk + 2 - C::STAGES : sk + 2;
@@ -342,12 +347,22 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 const int rr = rem / p.rope.gw;
                 const int col = rem - rr * p.rope.gw;
                 uint8_t* qrow = smem + C::OFF_Q + g * C::Q_TILE + row * 128;
+                // every (cos, sin) of the row first, as independent loads, then the
+                // rotation: interleaving the two serialises one table latency per chunk
+                float2 cs[D / 2];
+#pragma unroll
+                for (int i = 0; i < D / 2; ++i) cs[i] = rope_cs(p.rope, p.rope.t_tab, i, f, rr, col);
 #pragma unroll
                 for (int c = 0; c < D / 8; ++c) {
                     const int cb = c >> 3, cc = c & 7;
                     uint4* ptr = reinterpret_cast<uint4*>(qrow + cb * (kBM * 128) +
                                                           ((cc ^ (row & 7)) << 4));
-                    *ptr = rope_rotate8(*ptr, c * 8, f, rr, col, p.rope, p.rope.t_tab);
+                    uint4 v = *ptr;
+                    v.x = rope_pair(v.x, cs[4 * c + 0].x, cs[4 * c + 0].y);
+                    v.y = rope_pair(v.y, cs[4 * c + 1].x, cs[4 * c + 1].y);
+                    v.z = rope_pair(v.z, cs[4 * c + 2].x, cs[4 * c + 2].y);
+                    v.w = rope_pair(v.w, cs[4 * c + 3].x, cs[4 * c + 3].y);
+                    *ptr = v;
                 }
                 fence_proxy_async_smem();
             }
@@ -519,33 +534,49 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             named_bar_sync(1, 256);
             if (bars->last_split && store) {
                 __threadfence();
+                // unrolled over the largest split count so that every partial a column
+                // block needs is in flight at once (a runtime-bounded loop would wait one
+                // L2 round trip per split and per block)
                 const size_t prow0 = size_t(group) * p.n_split * 2 * kBM + g * kBM + row;
+                float2 ml[kMaxSplit];
+#pragma unroll
+                for (int r = 0; r < kMaxSplit; ++r)
+                    ml[r] = (r < p.n_split) ? __ldcg(&p.part_ml[prow0 + size_t(r) * 2 * kBM])
+                                            : make_float2(-INFINITY, 0.0f);
                 float mref = -INFINITY;
-                for (int r = 0; r < p.n_split; ++r)
-                    mref = fmaxf(mref, __ldcg(&p.part_ml[prow0 + size_t(r) * 2 * kBM]).x);
+#pragma unroll
+                for (int r = 0; r < kMaxSplit; ++r) mref = fmaxf(mref, ml[r].x);
+                float wr[kMaxSplit];
                 float lsum = 0.0f;
-                for (int r = 0; r < p.n_split; ++r) {
-                    const float2 ml = __ldcg(&p.part_ml[prow0 + size_t(r) * 2 * kBM]);
-                    lsum += ex2_approx(ml.x - mref) * ml.y;
+#pragma unroll
+                for (int r = 0; r < kMaxSplit; ++r) {
+                    wr[r] = (r < p.n_split) ? ex2_approx(ml[r].x - mref) : 0.0f;
+                    lsum += wr[r] * ml[r].y;
                 }
                 const float inv_l = 1.0f / lsum;
 #pragma unroll 1
                 for (int c = 0; c < D / 32; ++c) {
-                    float v[32];
+                    float4 x[kMaxSplit][8];
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) v[i] = 0.0f;
-                    for (int r = 0; r < p.n_split; ++r) {
-                        const float w = ex2_approx(
-                            __ldcg(&p.part_ml[prow0 + size_t(r) * 2 * kBM]).x - mref);
+                    for (int r = 0; r < kMaxSplit; ++r) {
                         const float4* src = reinterpret_cast<const float4*>(
                             p.part_o + (prow0 + size_t(r) * 2 * kBM) * D + c * 32);
 #pragma unroll
+                        for (int i = 0; i < 8; ++i)
+                            x[r][i] = (r < p.n_split) ? __ldcg(src + i)
+                                                      : make_float4(0.f, 0.f, 0.f, 0.f);
+                    }
+                    float v[32];
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] = 0.0f;
+#pragma unroll
+                    for (int r = 0; r < kMaxSplit; ++r) {
+#pragma unroll
                         for (int i = 0; i < 8; ++i) {
-                            const float4 x = __ldcg(src + i);
-                            v[4 * i] += w * x.x;
-                            v[4 * i + 1] += w * x.y;
-                            v[4 * i + 2] += w * x.z;
-                            v[4 * i + 3] += w * x.w;
+                            v[4 * i] += wr[r] * x[r][i].x;
+                            v[4 * i + 1] += wr[r] * x[r][i].y;
+                            v[4 * i + 2] += wr[r] * x[r][i].z;
+                            v[4 * i + 3] += wr[r] * x[r][i].w;
                         }
                     }
 #pragma unroll

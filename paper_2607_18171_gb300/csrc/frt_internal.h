@@ -45,14 +45,17 @@ __device__ __forceinline__ uint32_t rope_pair(uint32_t x, float c, float s) {
 }
 
 // t_tab: the chunk's t-segment table, either a.t_tab itself (parameter space) or a
-// shared-memory copy of it (kernels whose lanes index it divergently).
+// shared-memory copy of it (kernels whose lanes index it divergently). The h/w table is
+// read-only for the whole launch, so it is read through the non-coherent path: those
+// loads may then be issued ahead of the caller's stores of rotated values instead of
+// waiting behind each one.
 __device__ __forceinline__ float2 rope_cs(const RopeArgs& a, const float2* t_tab, int pi, int f,
                                           int r, int col) {
     if (pi < a.dt2) return t_tab[f * a.dt2 + pi];
     pi -= a.dt2;
-    if (pi < a.dh2) return a.hw[r * a.dh2 + pi];
+    if (pi < a.dh2) return __ldg(&a.hw[r * a.dh2 + pi]);
     pi -= a.dh2;
-    return a.hw[a.gh * a.dh2 + col * a.dw2 + pi];
+    return __ldg(&a.hw[a.gh * a.dh2 + col * a.dw2 + pi]);
 }
 
 // Rotate 8 consecutive head_dim elements [d0, d0+8) (d0 % 8 == 0) of a token at
