@@ -72,6 +72,7 @@ struct Bars {
     uint64_t kv_full[8];
     uint64_t step_done[4];
     uint64_t k0_done;
+    uint64_t epi_full[2];
     uint32_t tmem_base;
     int abort_flag;
     int last_split;
@@ -88,22 +89,6 @@ __device__ __forceinline__ void report(DeviceStatus* st, volatile int* abort, in
             __threadfence_system();
             s->code = kTimeoutCode;
         }
-    }
-}
-
-// 32 consecutive output values of one row -> fp32 or bf16 output
-__device__ __forceinline__ void store_row32(void* out, int out_bf16, size_t off, const float (&v)[32]) {
-    if (out_bf16) {
-        uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(out) + off);
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-            dst[i] = make_uint4(pack_bf16x2(v[8 * i + 0], v[8 * i + 1]), pack_bf16x2(v[8 * i + 2], v[8 * i + 3]),
-                                pack_bf16x2(v[8 * i + 4], v[8 * i + 5]), pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
-    } else {
-        float4* dst = reinterpret_cast<float4*>(static_cast<float*>(out) + off);
-#pragma unroll
-        for (int i = 0; i < 8; ++i)
-            dst[i] = make_float4(v[4 * i + 0], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
     }
 }
 
@@ -156,6 +141,8 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
         for (int s = 0; s < C::STAGES; ++s) mbar_init(smem_u32(&bars->kv_full[s]), 1);
         for (int s = 0; s < 4; ++s) mbar_init(smem_u32(&bars->step_done[s]), 1);
         mbar_init(smem_u32(&bars->k0_done), 1);
+        mbar_init(smem_u32(&bars->epi_full[0]), 1);
+        mbar_init(smem_u32(&bars->epi_full[1]), 1);
         bars->abort_flag = 0;
         fence_mbar_init();
         fence_proxy_async_smem();
@@ -347,11 +334,21 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 const int rr = rem / p.rope.gw;
                 const int col = rem - rr * p.rope.gw;
                 uint8_t* qrow = smem + C::OFF_Q + g * C::Q_TILE + row * 128;
-                // every (cos, sin) of the row first, as independent loads, then the
-                // rotation: interleaving the two serialises one table latency per chunk
+                // every (cos, sin) of the row first, then the rotation. Each entry is one
+                // load from an address chosen without branching (the t segment lives in
+                // the launch parameters, the h and w segments in the stream's table), so
+                // all of them are in flight together; a branch per entry on the runtime
+                // segment widths serialises one load latency per entry.
                 float2 cs[D / 2];
+                const int dt2 = p.rope.dt2, dth = p.rope.dt2 + p.rope.dh2;
+                const float2* t_row = p.rope.t_tab + f * dt2;
+                const float2* h_row = p.rope.hw + rr * p.rope.dh2 - dt2;
+                const float2* w_row = p.rope.hw + p.rope.gh * p.rope.dh2 + col * p.rope.dw2 - dth;
 #pragma unroll
-                for (int i = 0; i < D / 2; ++i) cs[i] = rope_cs(p.rope, p.rope.t_tab, i, f, rr, col);
+                for (int i = 0; i < D / 2; ++i) {
+                    const float2* src = i < dt2 ? t_row + i : (i < dth ? h_row + i : w_row + i);
+                    cs[i] = *src;
+                }
 #pragma unroll
                 for (int c = 0; c < D / 8; ++c) {
                     const int cb = c >> 3, cc = c & 7;
@@ -481,48 +478,95 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             mbar_arrive(smem_u32(&bars->p_full[g]));
         }
         // ---- epilogue ------------------------------------------------------------------
+        // O leaves through shared memory and TMA tensor stores. Once both tiles' last PV
+        // has completed the K/V ring is free: group g stages its 128-row tile in ring
+        // bytes [g * 512 * D, (g + 1) * 512 * D) as blocks of 128 rows x 128 bytes (32 fp32
+        // or 64 bf16 columns), 128-byte swizzled (16-byte chunk i of row r sits at chunk
+        // i ^ (r & 7)), which is the layout the tensor maps read. Rows past Nq are clipped
+        // by the store.
         if (ok) {
-            ok = __all_sync(0xffffffffu,
-                            mbar_wait(smem_u32(&bars->o_done[g]), 0, lim, abort));
+            bool got = mbar_wait(smem_u32(&bars->o_done[g]), 0, lim, abort);
+            if (got && ng == 2) got = mbar_wait(smem_u32(&bars->o_done[1 - g]), 0, lim, abort);
+            ok = __all_sync(0xffffffffu, got);
             if (!ok) report(p.status, abort, 2 + g, 4000);
         }
-        const bool store = ok && grow < sd.n_q;
-        const size_t obase = (size_t(grow) * p.heads + head) * D;
-        if (ok && p.n_split == 1) {
-            // O / l -> out
-            tc_fence_after();
-            const float inv_l = 1.0f / l_run;
+        const uint32_t stg = sKV + uint32_t(g * 512 * D);
+        const uint32_t sw = uint32_t(row & 7);
+        const bool leader = (sub == 0) && (lane == 0);    // issues the group's TMA copies
+        auto stage_f32 = [&](int c, const float (&v)[32]) {   // columns [32c, 32c + 32)
+            const uint32_t rb = stg + uint32_t(c * 16384 + row * 128);
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+                st_shared_v4(rb + ((uint32_t(i) ^ sw) << 4), __float_as_uint(v[4 * i]),
+                             __float_as_uint(v[4 * i + 1]), __float_as_uint(v[4 * i + 2]),
+                             __float_as_uint(v[4 * i + 3]));
+        };
+        auto stage_bf16 = [&](int c, const float (&v)[32]) {  // columns [32c, 32c + 32)
+            const uint32_t rb = stg + uint32_t((c >> 1) * 16384 + row * 128);
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                st_shared_v4(rb + ((uint32_t((c & 1) * 4 + i) ^ sw) << 4),
+                             pack_bf16x2(v[8 * i], v[8 * i + 1]), pack_bf16x2(v[8 * i + 2], v[8 * i + 3]),
+                             pack_bf16x2(v[8 * i + 4], v[8 * i + 5]), pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
+        };
+        // staged tile -> out (the group's leader); the CTA may exit once the reads are done
+        auto store_out = [&]() {
+            fence_proxy_async_smem();
+            named_bar_sync(2 + g, 128);
+            if (ok && leader) {
+                const int nb = p.out_bf16 ? D / 64 : D / 32;
+                for (int cb = 0; cb < nb; ++cb)
+                    tma_store_3d(&sd.out_map, stg + uint32_t(cb * 16384), cb * (p.out_bf16 ? 64 : 32),
+                                 head, m0 + g * kBM);
+                bulk_commit();
+                bulk_wait_read<0>();
+            }
+        };
+        if (p.n_split == 1) {
+            if (ok) {
+                // O / l -> out
+                tc_fence_after();
+                const float inv_l = 1.0f / l_run;
 #pragma unroll 1
-            for (int c = 0; c < D / 32; ++c) {
-                uint32_t o[32];
-                tmem_ld32(tO + c * 32, o);
-                tmem_ld_wait();
-                if (store) {
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t o[32];
+                    tmem_ld32(tO + c * 32, o);
+                    tmem_ld_wait();
                     float v[32];
 #pragma unroll
                     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(o[i]) * inv_l;
-                    store_row32(sd.out, p.out_bf16, obase + c * 32, v);
+                    if (p.out_bf16) stage_bf16(c, v);
+                    else stage_f32(c, v);
                 }
             }
-        } else if (ok) {
-            // unnormalised partial of this split -> scratch
-            tc_fence_after();
-            const size_t prow = (size_t(group) * p.n_split + split) * 2 * kBM + g * kBM + row;
-            float4* po = reinterpret_cast<float4*>(p.part_o + prow * D);
+            store_out();
+        } else {
+            // unnormalised partial of this split -> scratch (rows of tile (group, split, g))
+            const int prow_tile = int((size_t(group) * p.n_split + split) * 2 * kBM) + g * kBM;
+            if (ok) {
+                tc_fence_after();
 #pragma unroll 1
-            for (int c = 0; c < D / 32; ++c) {
-                uint32_t o[32];
-                tmem_ld32(tO + c * 32, o);
-                tmem_ld_wait();
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t o[32];
+                    tmem_ld32(tO + c * 32, o);
+                    tmem_ld_wait();
+                    float v[32];
 #pragma unroll
-                for (int i = 0; i < 8; ++i)
-                    po[c * 8 + i] = make_float4(__uint_as_float(o[4 * i]), __uint_as_float(o[4 * i + 1]),
-                                                __uint_as_float(o[4 * i + 2]), __uint_as_float(o[4 * i + 3]));
+                    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(o[i]);
+                    stage_f32(c, v);
+                }
+                p.part_ml[prow_tile + row] = make_float2(m_run, l_run);
             }
-            p.part_ml[prow] = make_float2(m_run, l_run);
+            fence_proxy_async_smem();
+            named_bar_sync(2 + g, 128);
+            if (ok && leader) {
+                for (int cb = 0; cb < D / 32; ++cb)
+                    tma_store_2d(&p.part_map, stg + uint32_t(cb * 16384), cb * 32, prow_tile);
+                bulk_commit();
+                bulk_wait<0>();   // written, not only read: other CTAs read it next
+                fence_proxy_async_global();
+            }
             __threadfence();
-        }
-        if (p.n_split > 1) {
             // the last split of this query group to finish merges all partials
             named_bar_sync(1, 256);
             if (threadIdx.x == 128) {
@@ -532,17 +576,16 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 bars->last_split = last;
             }
             named_bar_sync(1, 256);
-            if (bars->last_split && store) {
+            if (bars->last_split) {
                 __threadfence();
-                // unrolled over the largest split count so that every partial a column
-                // block needs is in flight at once (a runtime-bounded loop would wait one
-                // L2 round trip per split and per block)
-                const size_t prow0 = size_t(group) * p.n_split * 2 * kBM + g * kBM + row;
+                fence_proxy_async_global();
+                const int prow0 = int(size_t(group) * p.n_split * 2 * kBM) + g * kBM;
                 float2 ml[kMaxSplit];
 #pragma unroll
                 for (int r = 0; r < kMaxSplit; ++r)
-                    ml[r] = (r < p.n_split) ? __ldcg(&p.part_ml[prow0 + size_t(r) * 2 * kBM])
-                                            : make_float2(-INFINITY, 0.0f);
+                    ml[r] = (r == split) ? make_float2(m_run, l_run)
+                            : (r < p.n_split) ? __ldcg(&p.part_ml[prow0 + r * 2 * kBM + row])
+                                              : make_float2(-INFINITY, 0.0f);
                 float mref = -INFINITY;
 #pragma unroll
                 for (int r = 0; r < kMaxSplit; ++r) mref = fmaxf(mref, ml[r].x);
@@ -553,36 +596,78 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                     wr[r] = (r < p.n_split) ? ex2_approx(ml[r].x - mref) : 0.0f;
                     lsum += wr[r] * ml[r].y;
                 }
-                const float inv_l = 1.0f / lsum;
-#pragma unroll 1
-                for (int c = 0; c < D / 32; ++c) {
-                    float4 x[kMaxSplit][8];
+                const float w_own = ex2_approx(m_run - mref);
+                // splits are accumulated in index order whichever of them merges, so the
+                // result does not depend on which split finished last; this split's own O
+                // comes from TMEM, the others' through the group's staging
+                float v[D];
 #pragma unroll
-                    for (int r = 0; r < kMaxSplit; ++r) {
-                        const float4* src = reinterpret_cast<const float4*>(
-                            p.part_o + (prow0 + size_t(r) * 2 * kBM) * D + c * 32);
+                for (int i = 0; i < D; ++i) v[i] = 0.0f;
+                int phase = 0;
 #pragma unroll
-                        for (int i = 0; i < 8; ++i)
-                            x[r][i] = (r < p.n_split) ? __ldcg(src + i)
-                                                      : make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int r = 0; r < kMaxSplit; ++r) {
+                    if (r >= p.n_split) continue;
+                    if (r == split) {
+                        if (ok) {
+                            tc_fence_after();
+#pragma unroll
+                            for (int c = 0; c < D / 32; ++c) {
+                                uint32_t o[32];
+                                tmem_ld32(tO + c * 32, o);
+                                tmem_ld_wait();
+#pragma unroll
+                                for (int i = 0; i < 32; ++i)
+                                    v[c * 32 + i] += w_own * __uint_as_float(o[i]);
+                            }
+                        }
+                        continue;
                     }
-                    float v[32];
+                    const uint32_t fb = smem_u32(&bars->epi_full[g]);
+                    if (ok && leader) {
+                        mbar_arrive_expect_tx(fb, uint32_t(512 * D));
+                        for (int cb = 0; cb < D / 32; ++cb)
+                            tma_load_2d(stg + uint32_t(cb * 16384), &p.part_map, fb, cb * 32,
+                                        prow0 + r * 2 * kBM);
+                    }
+                    bool got = ok;
+                    if (got) {
+                        // the leader drains its own load even after an abort elsewhere
+                        got = leader ? mbar_wait_drain(fb, phase & 1, lim)
+                                     : mbar_wait(fb, phase & 1, lim, abort);
+                        got = __all_sync(0xffffffffu, got);
+                        if (!got) report(p.status, abort, 2 + g, 5000 + r);
+                    }
+                    ok = ok && got;
+                    if (ok) {
+                        const float w = wr[r];
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) v[i] = 0.0f;
+                        for (int c = 0; c < D / 32; ++c) {
+                            const uint32_t rb = stg + uint32_t(c * 16384 + row * 128);
 #pragma unroll
-                    for (int r = 0; r < kMaxSplit; ++r) {
-#pragma unroll
-                        for (int i = 0; i < 8; ++i) {
-                            v[4 * i] += wr[r] * x[r][i].x;
-                            v[4 * i + 1] += wr[r] * x[r][i].y;
-                            v[4 * i + 2] += wr[r] * x[r][i].z;
-                            v[4 * i + 3] += wr[r] * x[r][i].w;
+                            for (int i = 0; i < 8; ++i) {
+                                const uint4 x = ld_shared_v4(rb + ((uint32_t(i) ^ sw) << 4));
+                                v[c * 32 + 4 * i] += w * __uint_as_float(x.x);
+                                v[c * 32 + 4 * i + 1] += w * __uint_as_float(x.y);
+                                v[c * 32 + 4 * i + 2] += w * __uint_as_float(x.z);
+                                v[c * 32 + 4 * i + 3] += w * __uint_as_float(x.w);
+                            }
                         }
                     }
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) v[i] *= inv_l;
-                    store_row32(sd.out, p.out_bf16, obase + c * 32, v);
+                    ++phase;
+                    named_bar_sync(2 + g, 128);   // staging is refilled next
                 }
+                if (ok) {
+                    const float inv_l = 1.0f / lsum;
+#pragma unroll
+                    for (int c = 0; c < D / 32; ++c) {
+                        float x[32];
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) x[i] = v[c * 32 + i] * inv_l;
+                        if (p.out_bf16) stage_bf16(c, x);
+                        else stage_f32(c, x);
+                    }
+                }
+                store_out();
             }
         }
     }

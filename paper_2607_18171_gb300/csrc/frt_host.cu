@@ -72,6 +72,43 @@ frt_status make_map(CUtensorMap* map, const void* base, int head_dim, int heads,
     return FRT_OK;
 }
 
+// 3D map over an attention output [rows, heads, head_dim] (fp32 or bf16) for TMA stores:
+// box = 128 bytes of head_dim x 1 head x 128 rows, 128-byte swizzle; rows past `rows` are
+// not written.
+frt_status make_out_map(CUtensorMap* map, void* base, int head_dim, int heads, long long rows,
+                        bool bf16) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return fail(FRT_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+    const int es = bf16 ? 2 : 4;
+    cuuint64_t dims[3] = {cuuint64_t(head_dim), cuuint64_t(heads), cuuint64_t(rows)};
+    cuuint64_t strides[2] = {cuuint64_t(head_dim) * es, cuuint64_t(heads) * head_dim * es};
+    cuuint32_t box[3] = {cuuint32_t(128 / es), 1, 128};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = fn(map, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32,
+                    3, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                    CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(FRT_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", int(r));
+    return FRT_OK;
+}
+
+// 2D fp32 map over split-KV partial rows [rows, head_dim]: box 32 columns x 128 rows,
+// 128-byte swizzle (the layout the attention kernel stages its partial tiles in).
+frt_status make_part_map(CUtensorMap* map, float* base, int head_dim, long long rows) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return fail(FRT_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+    if (rows >= (1LL << 31)) return fail(FRT_ERR_UNSUPPORTED, "split-KV scratch too large");
+    cuuint64_t dims[2] = {cuuint64_t(head_dim), cuuint64_t(rows)};
+    cuuint64_t strides[1] = {cuuint64_t(head_dim) * 4};
+    cuuint32_t box[2] = {32, 128};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, base, dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(FRT_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", int(r));
+    return FRT_OK;
+}
+
 // 2D map over a row-major [rows, K] bf16 matrix; box = 64 columns x box_rows rows,
 // 128-byte swizzle; rows and columns past the extent read as zero.
 frt_status make_map_2d(CUtensorMap* map, const void* base, long long K, long long rows,
@@ -260,6 +297,13 @@ frt_status attention_single(frt_stream_t* s, const void* q, void* out, bool rope
     p.heads = s->heads;
     p.total_items = int(groups * p.n_split);
     p.out_bf16 = out_bf16 >= 0 ? out_bf16 : (s->cfg.out_dtype == FRT_OUT_BF16);
+    if ((st = make_out_map(&d.out_map, out, s->head_dim, s->heads, s->n_q, p.out_bf16 != 0)) !=
+        FRT_OK)
+        return st;
+    if (p.n_split > 1 &&
+        (st = make_part_map(&p.part_map, s->part_o, s->head_dim,
+                            s->part_groups * s->part_splits * 256)) != FRT_OK)
+        return st;
     p.scale_log2 = float(double(s->scale) * 1.4426950408889634);
     p.wait_limit_ns = s->wait_limit_ns;
     p.status = s->status_dev;
@@ -781,6 +825,11 @@ frt_status frt_chunk_attention_batched(frt_stream_t* const* streams, int n, cons
         return st;
     }
     p->n_split = n_split;
+    if (n_split > 1 && (st = make_part_map(&p->part_map, s0->part_o, s0->head_dim,
+                                           s0->part_groups * s0->part_splits * 256)) != FRT_OK) {
+        delete p;
+        return st;
+    }
     p->part_o = s0->part_o;
     p->part_ml = s0->part_ml;
     p->counters = s0->counters;
@@ -793,6 +842,11 @@ frt_status frt_chunk_attention_batched(frt_stream_t* const* streams, int n, cons
         if ((st = make_map(&d.q_map, q[i], s->head_dim, s->heads, s->n_q)) != FRT_OK ||
             (st = make_map(&d.k_map, s->cache_k, s->head_dim, s->heads, nkv)) != FRT_OK ||
             (st = make_map(&d.v_map, s->cache_v, s->head_dim, s->heads, nkv)) != FRT_OK) {
+            delete p;
+            return st;
+        }
+        if ((st = make_out_map(&d.out_map, out[i], s->head_dim, s->heads, s->n_q,
+                               s0->cfg.out_dtype == FRT_OUT_BF16)) != FRT_OK) {
             delete p;
             return st;
         }

@@ -78,6 +78,7 @@ struct AttnStreamDesc {
     CUtensorMap q_map;   // 3D (D, H, Nq), box (64, 1, 128), 128-byte swizzle
     CUtensorMap k_map;   // 3D (D, H, Nkv), box (64, 1, 128)
     CUtensorMap v_map;
+    CUtensorMap out_map; // 3D (D, H, Nq) over out: fp32 box (32, 1, 128) or bf16 box (64, 1, 128)
     void* out;           // [Nq, H, D] fp32 or bf16
     int n_q;
     int n_kv;
@@ -98,6 +99,7 @@ struct AttnParams {
     // processed by separate CTAs; each writes an unnormalised partial (O, running max,
     // row sum) and the last to finish merges them. n_split == 1 uses none of these.
     int n_split;
+    CUtensorMap part_map;        // 2D (D, groups * n_split * 256) fp32 over part_o, box (32, 128)
     float* part_o;               // [groups * n_split][2][128][D] fp32
     float2* part_ml;             // [groups * n_split][2][128] (max in log2 units, sum)
     int* counters;               // [groups], zero between launches

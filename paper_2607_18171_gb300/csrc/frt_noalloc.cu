@@ -37,7 +37,7 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
-bool encode(CUtensorMap* map, const void* base, int head_dim, int heads, long long rows) {
+EncodeTiledFn encode_fn() {
     static EncodeTiledFn fn = nullptr;
     static std::once_flag once;
     std::call_once(once, [] {
@@ -48,6 +48,12 @@ bool encode(CUtensorMap* map, const void* base, int head_dim, int heads, long lo
             q == cudaDriverEntryPointSuccess)
             fn = reinterpret_cast<EncodeTiledFn>(p);
     });
+    return fn;
+}
+
+// q/K/V: 3D (head_dim, heads, rows) bf16, box (64, 1, 128), 128-byte swizzle.
+bool encode(CUtensorMap* map, const void* base, int head_dim, int heads, long long rows) {
+    EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     cuuint64_t dims[3] = {cuuint64_t(head_dim), cuuint64_t(heads), cuuint64_t(rows)};
     cuuint64_t strides[2] = {cuuint64_t(head_dim) * 2, cuuint64_t(heads) * head_dim * 2};
@@ -57,6 +63,35 @@ bool encode(CUtensorMap* map, const void* base, int head_dim, int heads, long lo
               box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
            CUDA_SUCCESS;
+}
+
+// Output [rows, heads, head_dim] fp32 or bf16 for TMA stores: box of 128 bytes of head_dim
+// x 1 head x 128 rows, 128-byte swizzle.
+bool encode_out(CUtensorMap* map, void* base, int head_dim, int heads, long long rows, bool bf16) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    const int es = bf16 ? 2 : 4;
+    cuuint64_t dims[3] = {cuuint64_t(head_dim), cuuint64_t(heads), cuuint64_t(rows)};
+    cuuint64_t strides[2] = {cuuint64_t(head_dim) * es, cuuint64_t(heads) * head_dim * es};
+    cuuint32_t box[3] = {cuuint32_t(128 / es), 1, 128};
+    cuuint32_t estr[3] = {1, 1, 1};
+    return fn(map, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3,
+              base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+              CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Split-KV partial rows [rows, head_dim] fp32: box 32 x 128, 128-byte swizzle.
+bool encode_part(CUtensorMap* map, float* base, int head_dim, long long rows) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {cuuint64_t(head_dim), cuuint64_t(rows)};
+    cuuint64_t strides[1] = {cuuint64_t(head_dim) * 4};
+    cuuint32_t box[2] = {32, 128};
+    cuuint32_t estr[2] = {1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, base, dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 frt_status fail(frt_status st, const char* msg) {
@@ -131,6 +166,9 @@ extern "C" frt_status frt_chunk_attention_noalloc(const void* q, const void* k, 
     AttnStreamDesc& d = p.s[0];
     if (!encode(&d.q_map, q, head_dim, heads, n_q) || !encode(&d.k_map, k, head_dim, heads, n_kv) ||
         !encode(&d.v_map, v, head_dim, heads, n_kv))
+        return fail(FRT_ERR_CUDA, "tensor map encoding failed");
+    if (!encode_out(&d.out_map, out, head_dim, heads, n_q, out_dtype == FRT_OUT_BF16) ||
+        (split > 1 && !encode_part(&p.part_map, part_o, head_dim, (long long)groups * split * 256)))
         return fail(FRT_ERR_CUDA, "tensor map encoding failed");
     d.out = out;
     d.n_q = n_q;
