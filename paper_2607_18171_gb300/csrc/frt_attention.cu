@@ -229,8 +229,9 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             const uint64_t dk0 = sdesc_sw128(sKV, 16, 1024);
             const uint64_t dv0 = sdesc_sw128(sKV, kBN * 128, 1024);
             auto wait_load = [&](int Lw) -> bool {
-                if (!mbar_wait(smem_u32(&bars->kv_full[Lw % C::STAGES]), (Lw / C::STAGES) & 1,
-                               lim, abort)) {
+                const uint32_t fb = smem_u32(&bars->kv_full[Lw % C::STAGES]);
+                const uint32_t par = (Lw / C::STAGES) & 1;
+                if (!mbar_test_wait(fb, par) && !mbar_wait(fb, par, lim, abort)) {
                     report(p.status, abort, 1, Lw);
                     return false;
                 }
@@ -281,11 +282,28 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 umma_commit(smem_u32(&bars->k0_done));
             }
             int sv = 1 % C::STAGES, sk = 2 % C::STAGES;   // ring slots of V_j and K_{j+1}
+            // An MMA issue returns only once the previous MMA has drained, so a blocking
+            // wait at a group boundary idles the tensor pipe. P_g of the next PV group is
+            // therefore probed (non-blocking) from the shadow of the last MMAs of the
+            // group before it; when a probe has seen it complete, only the fence remains
+            // at the boundary.
+            auto take_p = [&](int g, int j, bool seen) -> bool {
+                if (seen) {
+                    tc_fence_after();
+                    return true;
+                }
+                return wait_p(g, j);
+            };
+            auto probe_p = [&](int g, int j) -> bool {
+                return mbar_test_wait(smem_u32(&bars->p_full[g]), j & 1);
+            };
+            bool p0_seen = false, p1_seen = false;
             for (int j = 0; j < n_tiles && ok; ++j) {
                 const bool more = (j + 1) < n_tiles;
                 // V_j has been waited for; K_{j+1} is waited for inside PV_0(j);
                 // V_{j+1} inside the last group of this step.
-                if (!(ok = wait_p(0, j))) break;
+                if (!(ok = take_p(0, j, p0_seen))) break;
+                p0_seen = false;
                 // the release of step j-1 rides in the shadow of PV_0(j)'s second MMA
                 // instead of idling the tensor pipe at the end of step j-1
                 issue_o(0, sv, j > 0, [&](int k) {
@@ -294,11 +312,15 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 });
                 if (!ok) break;
                 if (ng == 2) {
-                    if (more) issue_s(0, sk, nop);
+                    if (more) issue_s(0, sk, [&](int k) { if (k >= 5 && !p1_seen) p1_seen = probe_p(1, j); });
                     else umma_commit(smem_u32(&bars->o_done[0]));
-                    if (!(ok = wait_p(1, j))) break;
+                    if (!(ok = take_p(1, j, p1_seen))) break;
+                    p1_seen = false;
                     issue_o(1, sv, j > 0, nop);
-                    if (more) issue_s(1, sk, [&](int k) { if (k == 0) ok = wait_load(2 * j + 3); });
+                    if (more) issue_s(1, sk, [&](int k) {
+                        if (k == 0) ok = wait_load(2 * j + 3);
+                        if (k >= 5 && !p0_seen) p0_seen = probe_p(0, j + 1);
+                    });
                     else umma_commit(smem_u32(&bars->o_done[1]));
                 } else {
                     if (more) issue_s(0, sk, [&](int k) { if (k == 0) ok = wait_load(2 * j + 3); });
@@ -598,71 +620,88 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 }
                 const float w_own = ex2_approx(m_run - mref);
                 // splits are accumulated in index order whichever of them merges, so the
-                // result does not depend on which split finished last; this split's own O
-                // comes from TMEM, the others' through the group's staging
-                float v[D];
-#pragma unroll
-                for (int i = 0; i < D; ++i) v[i] = 0.0f;
+                // result does not depend on which split finished last: this split's own O
+                // comes from TMEM, the others' tiles through the group's staging, and the
+                // running sum lives in the group's S columns of TMEM (free by now)
+                const uint32_t tAcc = tS;
+                bool first = true;
                 int phase = 0;
 #pragma unroll
                 for (int r = 0; r < kMaxSplit; ++r) {
                     if (r >= p.n_split) continue;
-                    if (r == split) {
-                        if (ok) {
-                            tc_fence_after();
-#pragma unroll
-                            for (int c = 0; c < D / 32; ++c) {
+                    const bool own = (r == split);
+                    if (!own) {
+                        const uint32_t fb = smem_u32(&bars->epi_full[g]);
+                        if (ok && leader) {
+                            mbar_arrive_expect_tx(fb, uint32_t(512 * D));
+                            for (int cb = 0; cb < D / 32; ++cb)
+                                tma_load_2d(stg + uint32_t(cb * 16384), &p.part_map, fb, cb * 32,
+                                            prow0 + r * 2 * kBM);
+                        }
+                        bool got = ok;
+                        if (got) {
+                            // the leader drains its own load even after an abort elsewhere
+                            got = leader ? mbar_wait_drain(fb, phase & 1, lim)
+                                         : mbar_wait(fb, phase & 1, lim, abort);
+                            got = __all_sync(0xffffffffu, got);
+                            if (!got) report(p.status, abort, 2 + g, 5000 + r);
+                        }
+                        ok = ok && got;
+                        ++phase;
+                    }
+                    if (ok) {
+                        const float w = own ? w_own : wr[r];
+                        tc_fence_after();
+#pragma unroll 1
+                        for (int c = 0; c < D / 32; ++c) {
+                            float x[32];
+                            if (own) {
                                 uint32_t o[32];
                                 tmem_ld32(tO + c * 32, o);
                                 tmem_ld_wait();
 #pragma unroll
+                                for (int i = 0; i < 32; ++i) x[i] = __uint_as_float(o[i]);
+                            } else {
+                                const uint32_t rb = stg + uint32_t(c * 16384 + row * 128);
+#pragma unroll
+                                for (int i = 0; i < 8; ++i) {
+                                    const uint4 q4 = ld_shared_v4(rb + ((uint32_t(i) ^ sw) << 4));
+                                    x[4 * i] = __uint_as_float(q4.x);
+                                    x[4 * i + 1] = __uint_as_float(q4.y);
+                                    x[4 * i + 2] = __uint_as_float(q4.z);
+                                    x[4 * i + 3] = __uint_as_float(q4.w);
+                                }
+                            }
+                            uint32_t a[32];
+                            if (first) {
+#pragma unroll
+                                for (int i = 0; i < 32; ++i) a[i] = __float_as_uint(0.0f + w * x[i]);
+                            } else {
+                                tmem_ld32(tAcc + c * 32, a);
+                                tmem_ld_wait();
+#pragma unroll
                                 for (int i = 0; i < 32; ++i)
-                                    v[c * 32 + i] += w_own * __uint_as_float(o[i]);
+                                    a[i] = __float_as_uint(__uint_as_float(a[i]) + w * x[i]);
                             }
+                            tmem_st32(tAcc + c * 32, a);
                         }
-                        continue;
+                        tmem_st_wait();
+                        tc_fence_before();
                     }
-                    const uint32_t fb = smem_u32(&bars->epi_full[g]);
-                    if (ok && leader) {
-                        mbar_arrive_expect_tx(fb, uint32_t(512 * D));
-                        for (int cb = 0; cb < D / 32; ++cb)
-                            tma_load_2d(stg + uint32_t(cb * 16384), &p.part_map, fb, cb * 32,
-                                        prow0 + r * 2 * kBM);
-                    }
-                    bool got = ok;
-                    if (got) {
-                        // the leader drains its own load even after an abort elsewhere
-                        got = leader ? mbar_wait_drain(fb, phase & 1, lim)
-                                     : mbar_wait(fb, phase & 1, lim, abort);
-                        got = __all_sync(0xffffffffu, got);
-                        if (!got) report(p.status, abort, 2 + g, 5000 + r);
-                    }
-                    ok = ok && got;
-                    if (ok) {
-                        const float w = wr[r];
-#pragma unroll
-                        for (int c = 0; c < D / 32; ++c) {
-                            const uint32_t rb = stg + uint32_t(c * 16384 + row * 128);
-#pragma unroll
-                            for (int i = 0; i < 8; ++i) {
-                                const uint4 x = ld_shared_v4(rb + ((uint32_t(i) ^ sw) << 4));
-                                v[c * 32 + 4 * i] += w * __uint_as_float(x.x);
-                                v[c * 32 + 4 * i + 1] += w * __uint_as_float(x.y);
-                                v[c * 32 + 4 * i + 2] += w * __uint_as_float(x.z);
-                                v[c * 32 + 4 * i + 3] += w * __uint_as_float(x.w);
-                            }
-                        }
-                    }
-                    ++phase;
-                    named_bar_sync(2 + g, 128);   // staging is refilled next
+                    first = false;
+                    if (!own) named_bar_sync(2 + g, 128);   // staging is refilled next
                 }
                 if (ok) {
                     const float inv_l = 1.0f / lsum;
-#pragma unroll
+                    tc_fence_after();
+#pragma unroll 1
                     for (int c = 0; c < D / 32; ++c) {
+                        uint32_t a[32];
+                        tmem_ld32(tAcc + c * 32, a);
+                        tmem_ld_wait();
                         float x[32];
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) x[i] = v[c * 32 + i] * inv_l;
+                        for (int i = 0; i < 32; ++i) x[i] = __uint_as_float(a[i]) * inv_l;
                         if (p.out_bf16) stage_bf16(c, x);
                         else stage_f32(c, x);
                     }
