@@ -299,3 +299,52 @@ class OracleBlock:
         y = linear(bf16_round(o).reshape(o.shape[0], self.d), self.w_o)
         return {"q_rot": q_r, "k_rot": k_r, "v": v, "o": o, "y": y, "slot": slot,
                 "evicted": evicted}
+
+
+def causal_conv3d(x_ext, w, bias, kt: int, kh: int, kw: int) -> np.ndarray:
+    """Causal 3D convolution of channels-last frames in fp64.
+
+    ``x_ext`` [kt - 1 + F, H, W, Cin]: the kt - 1 frames before the chunk followed by the
+    chunk's F frames; ``w`` [kt * kh * kw, Cout, Cin] with tap index (dt * kh + dh) * kw
+    + dw; ``bias`` [Cout]. Output frame t (0..F-1) at (h, w):
+        y[t, h, w, o] = bias[o] + sum over dt, dh, dw, c of
+                        w[tap, o, c] * x_ext[t + dt, h + dh - kh // 2, w + dw - kw // 2, c],
+    with positions outside the frame read as zero (spatial zero padding, stride 1)."""
+    x_ext = np.asarray(x_ext, np.float64)
+    w = np.asarray(w, np.float64)
+    n_ext, H, W, cin = x_ext.shape
+    F = n_ext - (kt - 1)
+    cout = w.shape[1]
+    ph, pw = kh // 2, kw // 2
+    padded = np.zeros((n_ext, H + 2 * ph, W + 2 * pw, cin))
+    padded[:, ph:ph + H, pw:pw + W, :] = x_ext
+    y = np.broadcast_to(np.asarray(bias, np.float64), (F, H, W, cout)).copy()
+    for dt in range(kt):
+        for dh in range(kh):
+            for dw in range(kw):
+                tap = (dt * kh + dh) * kw + dw
+                win = padded[dt:dt + F, dh:dh + H, dw:dw + W, :]
+                y += win @ w[tap].T
+    return y
+
+
+class OracleConvStream:
+    """A streaming causal 3D convolution layer: the per-stream state is the last kt - 1
+    input frames (zeros before the first chunk), the kind of recurrent state a streaming
+    video VAE decoder carries from one batch to the next (the (V, V, 1) self-edge of the
+    DiT -> VAE pipeline, App. A.3)."""
+
+    def __init__(self, cin: int, cout: int, kt: int, kh: int, kw: int, grid_h: int,
+                 grid_w: int):
+        self.kt, self.kh, self.kw = kt, kh, kw
+        self.cache = np.zeros((kt - 1, grid_h, grid_w, cin))
+
+    def step(self, x, w, bias):
+        """One chunk of frames x [F, H, W, Cin]: output [F, H, W, Cout]; the cache then
+        holds the last kt - 1 frames of (cache, x)."""
+        x = np.asarray(x, np.float64)
+        x_ext = np.concatenate([self.cache, x], axis=0)
+        y = causal_conv3d(x_ext, w, bias, self.kt, self.kh, self.kw)
+        if self.kt > 1:
+            self.cache = x_ext[-(self.kt - 1):].copy()
+        return y
