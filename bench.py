@@ -407,6 +407,83 @@ def run_gpu_steps(args, wl, world, rank, local, dev, peak_tf, peak_kind):
     }
 
 
+CONV_METRIC = ("streaming causal 3D convolution (VAE-decoder layer) TFLOP/s per frame-chunk "
+               "at 1 GB300")
+
+
+def run_gpu_conv(args, cw, world, rank, local):
+    """One chunk through a streaming causal 3D convolution layer per step (frt_conv_step:
+    the convolution on the tensor cores, then the frame-cache update), inputs cycled
+    from a pool of distinct chunks."""
+    import torch
+    from paper_2607_18171_gb300 import frt, synth
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    frt.lib()
+    stream = torch.cuda.current_stream()
+    peak_tf, _, peak_kind = load_peaks()
+    st = frt.ConvStream(cw.cin, cw.cout, cw.kt, cw.kh, cw.kw, cw.grid_h, cw.grid_w, cw.frames)
+    w, b = (t.to(dev) for t in synth.conv_weights(cw))
+    pool = [synth.conv_chunk(cw, rank, i).to(dev) for i in range(POOL)]
+    ys = [st.new_out() for _ in range(2)]
+    flops = cw.flops()
+
+    def step(i):
+        st.step(pool[i % POOL], w, b, ys[i % 2])
+
+    for i in range(args.warmup):
+        step(i)
+    st.sync()
+    n = args.steps
+    ev = timing_events(n, stream)
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        t0.record(stream)
+        for i in range(n):
+            ev[i][0].record(stream)
+            step(args.warmup + i)
+            ev[i][1].record(stream)
+        t1.record(stream)
+        torch.cuda.synchronize()
+    st.sync()
+    elapsed = max_over_ranks(t0.elapsed_time(t1), world, dev)
+    step_ms = statistics.mean(a.elapsed_time(b_) for a, b_ in ev)
+    st.close()
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    if rank != 0:
+        return None
+    x_bytes = cw.frames * cw.grid_h * cw.grid_w * cw.cin * 2
+    return {
+        "metric": CONV_METRIC, "value": round(flops * n * world / (elapsed * 1e-3) / 1e12, 2),
+        "unit": UNIT, "n_gpus": world, "steps": n, "warmup": args.warmup,
+        "ms_per_step": round(elapsed / n, 4), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) channels-last frames, N(0,1/(taps*Cin)) weights)",
+        "config": {"workload": f"{cw.name}: Cin {cw.cin}, Cout {cw.cout}, kernel "
+                               f"{cw.kt}x{cw.kh}x{cw.kw} (causal in time, cache of "
+                               f"{cw.kt - 1} frames), {cw.grid_h}x{cw.grid_w} pixels, "
+                               f"{cw.frames} frames/chunk",
+                   "path": "frt_conv_step (implicit GEMM on tcgen05 + cache update: 2 launches)",
+                   "l2": f"{POOL} distinct chunks of {x_bytes / 1e6:.1f} MB cycled",
+                   "flops_per_step": flops},
+        "roofline": {"bound": "tensor", "achieved": round(flops / (step_ms * 1e-3) / 1e12, 2),
+                     "peak": peak_tf, "unit": "TFLOP/s",
+                     "frac": round(flops / (step_ms * 1e-3) / 1e12 / peak_tf, 4), "traffic": None,
+                     "kernel": "conv_kernel (+ cache_shift_kernel)", "peak_kind": peak_kind,
+                     "launch_ms": round(step_ms, 4)},
+        "clocks": clk.summary(),
+        "gpu_launches": (2 if cw.kt > 1 else 1) * n,
+    }
+
+
 BLOCK_METRIC = ("DiT-block attention-slice TFLOP/s (QKV projection + RoPE + KV append + "
                 "chunk attention + output projection) per frame-chunk at 1 GB300")
 
@@ -618,8 +695,13 @@ def main():
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     from paper_2607_18171_gb300 import synth
-    wl = synth.WORKLOADS[args.workload]
     world, rank, local = init_dist()
+    if args.workload in synth.CONV_WORKLOADS and args.impl != "reference":
+        line = run_gpu_conv(args, synth.CONV_WORKLOADS[args.workload], world, rank, local)
+        if line is not None:
+            print(json.dumps(line), flush=True)
+        return
+    wl = synth.WORKLOADS[args.workload]
     if args.impl == "reference":
         line = run_reference(args, wl, world, rank)
     else:

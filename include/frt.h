@@ -163,6 +163,40 @@ frt_status frt_gemm_bf16(const void* a, const void* b, void* c, int M, int N,
                          int K, int ldc, int c_dtype, void* status,
                          void* cuda_stream);
 
+/* ---- Streaming causal 3D convolution (the VAE-decoder stage) --------------------
+ * The paper's video pipelines end in a streaming VAE decoder (Appendix A.3, the
+ * DiT -> VAE template: the decoder carries state from one batch to the next, the
+ * (V, V, 1) self-edge). Its building block is a causal 3D convolution over a chunk
+ * of F frames whose kt - 1 temporal taps reach into a cache of the previous chunk's
+ * last frames (zeros before the first chunk). For output frame t, pixel (h, w),
+ * channel o:
+ *   y = bias[o] + sum over taps (dt, dh, dw), channels c of
+ *       w[(dt*kh + dh)*kw + dw][o][c] * x_ext[t + dt][h + dh - kh/2][w + dw - kw/2][c]
+ * with x_ext = (cache frames, chunk frames) and zeros outside the frame.
+ * Tensors are channels-last: x [F, H, W, Cin] bf16, w [kt*kh*kw, Cout, Cin] bf16,
+ * bias [Cout] fp32, y [F, H, W, Cout] fp32 or bf16; device pointers, 16-byte
+ * aligned, owned by the caller. A handle owns its frame cache (two [kt-1, H, W, Cin]
+ * bf16 buffers used in turn), allocated in frt_conv_configure. Cin and Cout are
+ * multiples of 64; 1 <= kt <= 4; kh, kw odd and <= 7. Not thread-safe per handle. */
+typedef struct frt_conv frt_conv_t;
+/* NULL on invalid sizes (frt_last_error()). */
+frt_conv_t* frt_conv_create(int cin, int cout, int kt, int kh, int kw, int grid_h,
+                            int grid_w, int frames_per_chunk);
+/* Allocate the cache (zeroed) and the status word; set the output dtype and the
+ * cudaStream_t every later call enqueues on. May be called again to change them. */
+frt_status frt_conv_configure(frt_conv_t* c, int out_dtype, void* cuda_stream);
+/* One chunk: y from (cache, x), then the cache becomes the last kt - 1 frames of
+ * (cache, x). Two launches (the convolution on the tensor cores, the cache update). */
+frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w,
+                         const void* bias, void* y);
+/* The current cache [kt-1, H, W, Cin] bf16 (device, read-only use). */
+frt_status frt_conv_cache(const frt_conv_t* c, const void** cache);
+/* Wait for the handle's work; returns FRT_ERR_TIMEOUT if a device wait gave up. */
+frt_status frt_conv_sync(frt_conv_t* c);
+/* Zero the cache and the status word (synchronises first). */
+frt_status frt_conv_reset(frt_conv_t* c);
+void frt_conv_destroy(frt_conv_t* c);
+
 /* Operation 3 for n independent streams in one launch (ragged KV lengths):
  * each streams[i] must have just appended (as for frt_chunk_attention); q[i]
  * and out[i] are that stream's rotated queries and output. All streams must

@@ -67,6 +67,13 @@ def lib() -> ctypes.CDLL:
         "frt_stream_set_append_events": (I, [P, P, P]),
         "frt_chunk_attention_noalloc": (I, [P, P, P, P, I, I, I, I, D, I, P, P]),
         "frt_block_step": (I, [P, P, P, P, P, P, P, ctypes.POINTER(I), ctypes.POINTER(LL)]),
+        "frt_conv_create": (P, [I, I, I, I, I, I, I, I]),
+        "frt_conv_configure": (I, [P, I, P]),
+        "frt_conv_step": (I, [P, P, P, P, P]),
+        "frt_conv_cache": (I, [P, ctypes.POINTER(P)]),
+        "frt_conv_sync": (I, [P]),
+        "frt_conv_reset": (I, [P]),
+        "frt_conv_destroy": (None, [P]),
         "frt_gemm_bf16": (I, [P, P, P, I, I, I, I, I, P, P]),
         "frt_stream_set_block_events": (I, [P, P, P, P, P]),
         "frt_window_index": (I, [LL, I, ctypes.POINTER(I), ctypes.POINTER(LL),
@@ -281,6 +288,60 @@ def _view_bf16(ptr: int, shape) -> torch.Tensor:
 
     t = torch.as_tensor(_Holder(), device="cuda")
     return t.view(torch.bfloat16).view(*shape)
+
+
+class ConvStream:
+    """A streaming causal 3D convolution layer (its frame cache lives in the library)."""
+
+    def __init__(self, cin: int, cout: int, kt: int, kh: int, kw: int, grid_h: int,
+                 grid_w: int, frames_per_chunk: int, out_dtype: torch.dtype = torch.float32,
+                 cuda_stream: torch.cuda.Stream | None = None):
+        L = lib()
+        self._h = L.frt_conv_create(cin, cout, kt, kh, kw, grid_h, grid_w, frames_per_chunk)
+        if not self._h:
+            raise FrtError(1, L.frt_last_error().decode())
+        self.cin, self.cout, self.kt, self.kh, self.kw = cin, cout, kt, kh, kw
+        self.grid_h, self.grid_w, self.frames = grid_h, grid_w, frames_per_chunk
+        self.out_dtype = out_dtype
+        self.torch_stream = cuda_stream or torch.cuda.current_stream()
+        _check(L.frt_conv_configure(self._h, OUT_BF16 if out_dtype == torch.bfloat16 else OUT_F32,
+                                    ctypes.c_void_p(self.torch_stream.cuda_stream)))
+
+    def new_out(self) -> torch.Tensor:
+        return torch.empty(self.frames, self.grid_h, self.grid_w, self.cout, dtype=self.out_dtype,
+                           device="cuda")
+
+    def step(self, x: torch.Tensor, w: torch.Tensor, bias: torch.Tensor, y: torch.Tensor) -> None:
+        _bf16_dev(x, (self.frames, self.grid_h, self.grid_w, self.cin), "x")
+        _bf16_dev(w, (self.kt * self.kh * self.kw, self.cout, self.cin), "w")
+        if bias.dtype != torch.float32 or not bias.is_cuda or tuple(bias.shape) != (self.cout,):
+            raise ValueError("bias must be a float32 CUDA tensor [Cout]")
+        if y.dtype != self.out_dtype or not y.is_cuda or not y.is_contiguous() or \
+                tuple(y.shape) != (self.frames, self.grid_h, self.grid_w, self.cout):
+            raise ValueError("y must be a contiguous [F, H, W, Cout] CUDA tensor of the out dtype")
+        _check(lib().frt_conv_step(self._h, _ptr(x), _ptr(w), _ptr(bias), _ptr(y)))
+
+    def cache(self) -> torch.Tensor:
+        p = ctypes.c_void_p()
+        _check(lib().frt_conv_cache(self._h, ctypes.byref(p)))
+        return _view_bf16(p.value, (max(1, self.kt - 1), self.grid_h, self.grid_w, self.cin))
+
+    def sync(self) -> None:
+        _check(lib().frt_conv_sync(self._h))
+
+    def reset(self) -> None:
+        _check(lib().frt_conv_reset(self._h))
+
+    def close(self) -> None:
+        if getattr(self, "_h", None):
+            lib().frt_conv_destroy(self._h)
+            self._h = None
+
+    def __del__(self):  # pragma: no cover - best effort
+        try:
+            self.close()
+        except Exception:
+            pass
 
 
 def chunk_attention_batched(streams, qs, outs) -> None:

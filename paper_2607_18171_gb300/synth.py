@@ -17,7 +17,9 @@ U(0.5, 2) once per stream (SeedSequence([1000*w + s, 999999])), then rounded
 to bf16 (round to nearest even). Ragged multi-stream fills are drawn
 uniform on {1..W} from SeedSequence([1000*w, 777777]). DiT-block workloads
 draw hidden states x ~ N(0, 1) [Nq, heads*head_dim] per chunk and projection
-weights ~ N(0, 1/d) once per workload (``chunk_x``, ``block_weights``).
+weights ~ N(0, 1/d) once per workload (``chunk_x``, ``block_weights``). Streaming
+convolution workloads (``CONV_WORKLOADS``) draw channels-last frames ~ N(0, 1) per chunk
+and weights ~ N(0, 1/(taps*Cin)) with a small bias (``conv_chunk``, ``conv_weights``).
 """
 
 from __future__ import annotations
@@ -139,6 +141,58 @@ def chunk_x(wl: Workload, stream: int, chunk: int) -> torch.Tensor:
     rng = np.random.Generator(np.random.PCG64(
         np.random.SeedSequence([1000 * wl.index + stream, chunk, 1])))
     return torch.from_numpy(rng.standard_normal((wl.n_q, d), dtype=np.float32)).to(torch.bfloat16)
+
+
+@dataclasses.dataclass(frozen=True)
+class ConvWorkload:
+    """A streaming causal 3D convolution layer of a video VAE decoder."""
+    name: str
+    index: int
+    cin: int
+    cout: int
+    kt: int
+    kh: int
+    kw: int
+    grid_h: int
+    grid_w: int
+    frames: int              # frames per chunk
+    chunks: int
+
+    @property
+    def taps(self) -> int:
+        return self.kt * self.kh * self.kw
+
+    def flops(self) -> int:
+        """2 * outputs * Cout * taps * Cin per chunk (one multiply-add = 2 flops)."""
+        return 2 * self.frames * self.grid_h * self.grid_w * self.cout * self.taps * self.cin
+
+
+CONV_WORKLOADS = {
+    "convtiny": ConvWorkload("convtiny", 20, 64, 64, 3, 3, 3, 5, 9, 2, 4),
+    # decoder layers of a 3-frame chunk: latent grid 30 x 52 at 384 channels, and the
+    # 2x upsampled 60 x 104 grid at 192 channels
+    "vae30x52c384": ConvWorkload("vae30x52c384", 21, 384, 384, 3, 3, 3, 30, 52, 3, 4),
+    "vae60x104c192": ConvWorkload("vae60x104c192", 22, 192, 192, 3, 3, 3, 60, 104, 3, 4),
+}
+
+
+def conv_weights(cw: ConvWorkload):
+    """(w [taps, Cout, Cin] bf16, bias [Cout] fp32): w ~ N(0, 1/(taps*Cin)), bias ~
+    N(0, 0.1^2), from PCG64(SeedSequence([1000*w, 444444]))."""
+    rng = np.random.Generator(np.random.PCG64(np.random.SeedSequence([1000 * cw.index, 444444])))
+    sd = np.float32(1.0 / math.sqrt(cw.taps * cw.cin))
+    w = rng.standard_normal((cw.taps, cw.cout, cw.cin), dtype=np.float32) * sd
+    b = rng.standard_normal(cw.cout, dtype=np.float32) * np.float32(0.1)
+    return torch.from_numpy(w).to(torch.bfloat16), torch.from_numpy(b)
+
+
+def conv_chunk(cw: ConvWorkload, stream: int, chunk: int) -> torch.Tensor:
+    """Chunk of input frames [F, H, W, Cin] bf16, N(0, 1), from
+    PCG64(SeedSequence([1000*w + stream, chunk, 2]))."""
+    rng = np.random.Generator(np.random.PCG64(
+        np.random.SeedSequence([1000 * cw.index + stream, chunk, 2])))
+    x = rng.standard_normal((cw.frames, cw.grid_h, cw.grid_w, cw.cin), dtype=np.float32)
+    return torch.from_numpy(x).to(torch.bfloat16)
 
 
 def as_f64(t: torch.Tensor) -> np.ndarray:

@@ -1,0 +1,142 @@
+"""GPU parity of the streaming causal 3D convolution (frt_conv_step) against the fp64
+oracle, through the C ABI: every output element at small sizes (ragged against the
+16 x 8 pixel tiles), sampled outputs at the VAE-decoder sizes, the frame cache
+bit-exact, determinism and the bf16 output.
+
+Tolerance: fp32 accumulation of K = taps * Cin bf16 products, whatever the order, is
+within K * 2^-24 * sum |w x| of the exact sum (tested with K * 2^-23 plus 1e-6); a bf16
+output adds half an ulp of the result."""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle.frt_oracle import OracleConvStream, causal_conv3d
+from paper_2607_18171_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def frt():
+    from paper_2607_18171_gb300 import frt as f
+    f.lib()
+    return f
+
+
+def _f64(t):
+    return t.detach().float().cpu().numpy().astype(np.float64)
+
+
+def _bound(cw, x_ext, w, out_bf16, ref):
+    """Elementwise error bound: K * 2^-23 * (|x_ext| conv |w|) (+ bf16 half ulp)."""
+    mag = causal_conv3d(np.abs(x_ext), np.abs(w), np.zeros(cw.cout), cw.kt, cw.kh, cw.kw)
+    b = cw.taps * cw.cin * 2.0 ** -23 * mag + 1e-6
+    if out_bf16:
+        b = b + 2.0 ** -8 * np.abs(ref)
+    return b
+
+
+SMALL = {
+    "convtiny": synth.CONV_WORKLOADS["convtiny"],
+    # ragged against the tiles, kt = 2 and kh != kw, two k-blocks of channels
+    "conv_ragged": synth.ConvWorkload("conv_ragged", 23, 128, 64, 2, 3, 5, 11, 21, 3, 3),
+    # one frame per chunk (the cache is shifted, not replaced), 256-wide N tiles
+    "conv_f1": synth.ConvWorkload("conv_f1", 24, 64, 256, 3, 3, 3, 9, 17, 1, 4),
+    # no temporal taps: nothing cached
+    "conv_kt1": synth.ConvWorkload("conv_kt1", 25, 64, 192, 1, 3, 3, 8, 16, 2, 2),
+}
+
+
+@pytest.mark.parametrize("name", list(SMALL))
+@pytest.mark.parametrize("out", [torch.float32, torch.bfloat16])
+def test_conv_stream_matches_oracle_every_element(frt, name, out):
+    cw = SMALL[name]
+    w, b = synth.conv_weights(cw)
+    wd, bd = w.cuda(), b.cuda()
+    st = frt.ConvStream(cw.cin, cw.cout, cw.kt, cw.kh, cw.kw, cw.grid_h, cw.grid_w, cw.frames,
+                        out_dtype=out)
+    orc = OracleConvStream(cw.cin, cw.cout, cw.kt, cw.kh, cw.kw, cw.grid_h, cw.grid_w)
+    wf, bf = synth.as_f64(w), b.double().numpy()
+    for c in range(cw.chunks):
+        x = synth.conv_chunk(cw, 0, c)
+        y = st.new_out()
+        st.step(x.cuda(), wd, bd, y)
+        st.sync()
+        x_ext = np.concatenate([orc.cache, synth.as_f64(x)], axis=0)
+        ref = orc.step(synth.as_f64(x), wf, bf)
+        got = _f64(y)
+        bound = _bound(cw, x_ext, wf, out == torch.bfloat16, ref)
+        err = np.abs(got - ref)
+        assert np.all(err <= bound), f"{name} chunk {c}: max excess {float(np.max(err - bound)):.3e}"
+        if cw.kt > 1:
+            assert np.array_equal(_f64(st.cache()), orc.cache), f"{name} chunk {c}: cache"
+    st.close()
+
+
+@pytest.mark.parametrize("name", ["vae30x52c384", "vae60x104c192"])
+def test_conv_vae_sizes_on_sampled_pixels(frt, name):
+    """Full VAE-decoder sizes: 4 chunks streamed; every output channel of 300 sampled
+    pixels (tile edges, frame borders, random) against the oracle's definition."""
+    cw = synth.CONV_WORKLOADS[name]
+    w, b = synth.conv_weights(cw)
+    st = frt.ConvStream(cw.cin, cw.cout, cw.kt, cw.kh, cw.kw, cw.grid_h, cw.grid_w, cw.frames)
+    wf, bf = synth.as_f64(w), b.double().numpy()
+    rng = np.random.default_rng(5)
+    cache = np.zeros((cw.kt - 1, cw.grid_h, cw.grid_w, cw.cin))
+    for c in range(cw.chunks):
+        x = synth.conv_chunk(cw, 0, c)
+        y = st.new_out()
+        st.step(x.cuda(), w.cuda(), b.cuda(), y)
+        st.sync()
+        xf = synth.as_f64(x)
+        x_ext = np.concatenate([cache, xf], axis=0)
+        got = _f64(y)
+        pix = [(t, h, ww) for t in range(cw.frames) for h in (0, 7, 8, cw.grid_h - 1)
+               for ww in (0, 15, 16, cw.grid_w - 1)]
+        pix += [(int(rng.integers(cw.frames)), int(rng.integers(cw.grid_h)),
+                 int(rng.integers(cw.grid_w))) for _ in range(300 - len(pix))]
+        ph, pw = cw.kh // 2, cw.kw // 2
+        pad = np.zeros((x_ext.shape[0], cw.grid_h + 2 * ph, cw.grid_w + 2 * pw, cw.cin))
+        pad[:, ph:ph + cw.grid_h, pw:pw + cw.grid_w] = x_ext
+        for (t, h, ww) in pix:
+            win = pad[t:t + cw.kt, h:h + cw.kh, ww:ww + cw.kw].reshape(cw.taps, cw.cin)
+            ref = bf + np.einsum("koc,kc->o", wf, win)
+            mag = np.einsum("koc,kc->o", np.abs(wf), np.abs(win))
+            err = np.abs(got[t, h, ww] - ref)
+            assert np.all(err <= cw.taps * cw.cin * 2.0 ** -23 * mag + 1e-6), (name, c, t, h, ww)
+        cache = x_ext[-(cw.kt - 1):]
+        assert np.array_equal(_f64(st.cache()), cache)
+    st.close()
+
+
+def test_conv_is_deterministic_and_reset_restarts(frt):
+    cw = SMALL["conv_ragged"]
+    w, b = (t.cuda() for t in synth.conv_weights(cw))
+    st = frt.ConvStream(cw.cin, cw.cout, cw.kt, cw.kh, cw.kw, cw.grid_h, cw.grid_w, cw.frames)
+    runs = []
+    for _ in range(2):
+        outs = []
+        for c in range(3):
+            y = st.new_out()
+            st.step(synth.conv_chunk(cw, 1, c).cuda(), w, b, y)
+            outs.append(y)
+        st.sync()
+        runs.append(outs)
+        st.reset()
+    for a, b_ in zip(*runs):
+        assert torch.equal(a, b_)
+    st.close()
+
+
+def test_conv_rejects_bad_arguments(frt):
+    with pytest.raises(frt.FrtError):
+        frt.ConvStream(48, 64, 3, 3, 3, 8, 8, 2)          # Cin not a multiple of 64
+    with pytest.raises(frt.FrtError):
+        frt.ConvStream(64, 64, 3, 2, 3, 8, 8, 2)          # even kh
+    cw = SMALL["convtiny"]
+    st = frt.ConvStream(cw.cin, cw.cout, cw.kt, cw.kh, cw.kw, cw.grid_h, cw.grid_w, cw.frames)
+    w, b = (t.cuda() for t in synth.conv_weights(cw))
+    with pytest.raises(ValueError):
+        st.step(torch.zeros(1, 2, 3, 64, dtype=torch.bfloat16, device="cuda"), w, b, st.new_out())
+    st.close()
