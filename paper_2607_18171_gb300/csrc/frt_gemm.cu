@@ -11,6 +11,11 @@
 //               tcgen05.ld.
 // The accumulator is double-buffered in TMEM (2 x BN columns), so the epilogue of tile i
 // runs while the tensor pipe computes tile i + 1.
+// With a cluster of CM = 2 CTAs the two work on adjacent M tiles of the same N tile and
+// share B: each loads its own A and one half of the B box, multicast into both CTAs'
+// shared memory, which halves the L2 reads of B (the kernel is bound by how fast L2 feeds
+// the SMs). A stage is refilled only after both CTAs' MMAs have read it: the MMA commit
+// that releases it is multicast to both CTAs' `empty` barriers.
 //
 // Epilogues:
 //   plain  C row-major, fp32 or bf16 (round to nearest even), rows >= M and columns >= N
@@ -71,9 +76,11 @@ __device__ __forceinline__ void report(DeviceStatus* st, volatile int* abort, in
     }
 }
 
-template <int BN>
+template <int BN, int CM>
 __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant__ GemmParams p) {
     using C = GCfg<BN>;
+    constexpr int B_SLICE = C::B_BYTES / CM;        // bytes of B this CTA loads
+    constexpr uint16_t kMask = uint16_t((1u << CM) - 1);
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
@@ -83,14 +90,19 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
     volatile int* abort = &bars.abort_flag;
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int n_tiles = p.tiles_m * p.tiles_n;
+    // cluster tiles: CM consecutive M tiles of one N tile
+    const int ctm = (p.tiles_m + CM - 1) / CM;
+    const int n_tiles = ctm * p.tiles_n;
+    const int rank = CM > 1 ? int(cluster_ctarank()) : 0;
+    const int c_first = blockIdx.x / CM;
+    const int c_stride = gridDim.x / CM;
     const int nk = (p.K + kBK - 1) / kBK;
     const uint64_t lim = p.wait_limit_ns;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(smem_u32(&bars.full[s]), 1);
-            mbar_init(smem_u32(&bars.empty[s]), 1);
+            mbar_init(smem_u32(&bars.empty[s]), CM);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&bars.acc_full[b]), 1);
@@ -108,6 +120,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
     }
     tc_fence_before();
     __syncthreads();
+    if (CM > 1) cluster_sync_all();   // every CTA's barriers exist before any multicast
     tc_fence_after();
     const uint32_t tmem = bars.tmem_base;
 
@@ -118,9 +131,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
             tma_prefetch_map(&p.b_map);
             int it = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
-                const int tm = t % p.tiles_m;
-                const int tn = t / p.tiles_m;
+            for (int t = c_first; t < n_tiles && ok; t += c_stride) {
+                const int tm = (t % ctm) * CM + rank;
+                const int tn = t / ctm;
                 for (int kb = 0; kb < nk; ++kb) {
                     const int s = it % kStages;
                     // slot s was last filled by load it - kStages; the MMA that read it
@@ -135,7 +148,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
                     mbar_arrive_expect_tx(fb, C::STAGE);
                     const uint32_t dst = sbase + s * C::STAGE;
                     tma_load_2d(dst, &p.a_map, fb, kb * kBK, tm * kBM);
-                    tma_load_2d(dst + C::A_BYTES, &p.b_map, fb, kb * kBK, tn * BN);
+                    if (CM == 1)
+                        tma_load_2d(dst + C::A_BYTES, &p.b_map, fb, kb * kBK, tn * BN);
+                    else
+                        tma_load_2d_mc(dst + C::A_BYTES + rank * B_SLICE, &p.b_map, fb, kb * kBK,
+                                       tn * BN + rank * (BN / CM), kMask);
                     ++it;
                 }
             }
@@ -153,7 +170,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
             int it = 0;
             int tl = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++tl) {
+            for (int t = c_first; t < n_tiles && ok; t += c_stride, ++tl) {
                 const int b = tl & 1;
                 if (tl >= 2 &&
                     !mbar_wait(smem_u32(&bars.acc_empty[b]), ((tl >> 1) - 1) & 1, lim, abort)) {
@@ -176,7 +193,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
                     for (int k = 0; k < kBK / 16; ++k)
                         umma_ss(d, da0 + so + uint64_t(2 * k), db0 + so + uint64_t(2 * k), C::IDESC,
                                 (kb > 0 || k > 0) ? 1u : 0u);
-                    umma_commit(smem_u32(&bars.empty[s]));
+                    if (CM == 1) umma_commit(smem_u32(&bars.empty[s]));
+                    else umma_commit_mc(smem_u32(&bars.empty[s]), kMask);
                 }
                 if (ok) umma_commit(smem_u32(&bars.acc_full[b]));
             }
@@ -190,10 +208,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
         const int row = sub * 32 + lane;
         const uint32_t lane_off = uint32_t(sub * 32) << 16;
         int tl = 0;
-        for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++tl) {
+        for (int t = c_first; t < n_tiles; t += c_stride, ++tl) {
             const int b = tl & 1;
-            const int tm = t % p.tiles_m;
-            const int tn = t / p.tiles_m;
+            const int tm = (t % ctm) * CM + rank;
+            const int tn = t / ctm;
             const bool got = mbar_wait(smem_u32(&bars.acc_full[b]), (tl >> 1) & 1, lim, abort);
             if (!__all_sync(0xffffffffu, got)) {
                 if (!got) report(p.status, abort, 2, tl);
@@ -290,27 +308,46 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
     __syncwarp();
     tc_fence_before();
     __syncthreads();
+    if (CM > 1) cluster_sync_all();   // no peer multicasts into or signals this CTA any more
     tc_fence_after();
     if (warp == 1) tmem_dealloc(tmem, C::TMEM_COLS);
 }
 
-template <int BN>
+template <int BN, int CM>
 cudaError_t launch(const GemmParams& p, cudaStream_t st) {
     static bool attr_set = false;
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(gemm_kernel<BN>,
+        cudaError_t e = cudaFuncSetAttribute(gemm_kernel<BN, CM>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              GCfg<BN>::SMEM);
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    const int n_tiles = p.tiles_m * p.tiles_n;
-    const int grid = n_tiles < num_sms() ? n_tiles : num_sms();
-    gemm_kernel<BN><<<grid, kThreads, GCfg<BN>::SMEM, st>>>(p);
-    return cudaGetLastError();
+    const int n_ctiles = ((p.tiles_m + CM - 1) / CM) * p.tiles_n;
+    const int clusters = n_ctiles < num_sms() / CM ? n_ctiles : num_sms() / CM;
+    if (CM == 1) {
+        gemm_kernel<BN, 1><<<clusters, kThreads, GCfg<BN>::SMEM, st>>>(p);
+        return cudaGetLastError();
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(unsigned(clusters * CM));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = GCfg<BN>::SMEM;
+    cfg.stream = st;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = CM;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, gemm_kernel<BN, CM>, p);
 }
 
 }  // namespace
+
+// CTAs per cluster sharing B: 2 whenever there are at least two M tiles.
+int gemm_cluster_m(int M) { return M > kBM ? 2 : 1; }
 
 int gemm_block_n(int N, int epi, int d) {
     // BN = 256 unless the QKV epilogue needs 128-column tiles (d not a multiple of 256)
@@ -324,7 +361,8 @@ cudaError_t launch_gemm(GemmParams p, cudaStream_t st) {
     const int bn = gemm_block_n(p.N, p.epi, p.d);
     p.tiles_m = (p.M + kBM - 1) / kBM;
     p.tiles_n = (p.N + bn - 1) / bn;
-    return bn == 256 ? launch<256>(p, st) : launch<128>(p, st);
+    if (gemm_cluster_m(p.M) == 2) return bn == 256 ? launch<256, 2>(p, st) : launch<128, 2>(p, st);
+    return bn == 256 ? launch<256, 1>(p, st) : launch<128, 1>(p, st);
 }
 
 }  // namespace frt

@@ -637,7 +637,8 @@ frt_status frt_block_step(frt_stream_t* s, const void* x, const void* w_qkv, con
     std::memset(&g, 0, sizeof(g));
     const int bn = gemm_block_n(3 * d, kEpiQkv, d);
     if ((st = make_map_2d(&g.a_map, x, d, s->n_q, 128)) != FRT_OK) return st;
-    if ((st = make_map_2d(&g.b_map, w_qkv, d, 3LL * d, bn)) != FRT_OK) return st;
+    if ((st = make_map_2d(&g.b_map, w_qkv, d, 3LL * d, bn / gemm_cluster_m(s->n_q))) != FRT_OK)
+        return st;
     g.M = s->n_q;
     g.N = 3 * d;
     g.K = d;
@@ -672,7 +673,7 @@ frt_status frt_block_step(frt_stream_t* s, const void* x, const void* w_qkv, con
     std::memset(&h, 0, sizeof(h));
     const int bn2 = gemm_block_n(d, kEpiPlain, 0);
     if ((st = make_map_2d(&h.a_map, o_buf, d, s->n_q, 128)) != FRT_OK) return st;
-    if ((st = make_map_2d(&h.b_map, w_o, d, d, bn2)) != FRT_OK) return st;
+    if ((st = make_map_2d(&h.b_map, w_o, d, d, bn2 / gemm_cluster_m(s->n_q))) != FRT_OK) return st;
     h.M = s->n_q;
     h.N = d;
     h.K = d;
@@ -705,7 +706,9 @@ frt_status frt_gemm_bf16(const void* a, const void* b, void* c, int M, int N, in
     std::memset(&g, 0, sizeof(g));
     frt_status st;
     if ((st = make_map_2d(&g.a_map, a, K, M, 128)) != FRT_OK) return st;
-    if ((st = make_map_2d(&g.b_map, b, K, N, gemm_block_n(N, kEpiPlain, 0))) != FRT_OK) return st;
+    if ((st = make_map_2d(&g.b_map, b, K, N, gemm_block_n(N, kEpiPlain, 0) / gemm_cluster_m(M))) !=
+        FRT_OK)
+        return st;
     g.M = M;
     g.N = N;
     g.K = K;
