@@ -11,11 +11,13 @@
 //               tcgen05.ld.
 // The accumulator is double-buffered in TMEM (2 x BN columns), so the epilogue of tile i
 // runs while the tensor pipe computes tile i + 1.
-// With a cluster of CM = 2 CTAs the two work on adjacent M tiles of the same N tile and
-// share B: each loads its own A and one half of the B box, multicast into both CTAs'
-// shared memory, which halves the L2 reads of B (the kernel is bound by how fast L2 feeds
-// the SMs). A stage is refilled only after both CTAs' MMAs have read it: the MMA commit
-// that releases it is multicast to both CTAs' `empty` barriers.
+// When M spans more than one 128-row tile, two CTAs of a cluster work as a pair on a
+// 256 x BN tile with tcgen05.mma.cta_group::2: each holds its own 128 rows of A and one
+// half of B in shared memory (the tensor cores of the two SMs read both halves), so each
+// SM takes in 32 KB per k-block instead of 48 — what bounds this kernel is how fast
+// operands reach an SM. The leader CTA's thread issues the MMAs for both; both CTAs'
+// TMA loads complete on the leader's barriers; the leader's commits reach both CTAs; the
+// follower's epilogue hands the accumulator back to the leader by a remote arrive.
 //
 // Epilogues:
 //   plain  C row-major, fp32 or bf16 (round to nearest even), rows >= M and columns >= N
@@ -39,22 +41,24 @@ namespace {
 constexpr int kThreads = 192;
 constexpr int kBM = 128;
 constexpr int kBK = 64;          // one 128-byte swizzle atom of bf16
-constexpr int kStages = 4;
+constexpr int kMaxStages = 6;
 constexpr int kTimeoutCode = 6;  // FRT_ERR_TIMEOUT
 
-template <int BN>
+template <int BN, bool PAIR>
 struct GCfg {
-    static constexpr int A_BYTES = kBM * kBK * 2;
-    static constexpr int B_BYTES = BN * kBK * 2;
+    static constexpr int CM = PAIR ? 2 : 1;               // CTAs per tile
+    static constexpr int A_BYTES = kBM * kBK * 2;         // this CTA's 128 rows of A
+    static constexpr int B_BYTES = (BN / CM) * kBK * 2;   // this CTA's share of B
     static constexpr int STAGE = A_BYTES + B_BYTES;
-    static constexpr int SMEM = kStages * STAGE + 1024;   // + alignment slack
-    static constexpr uint32_t IDESC = idesc_bf16_f32(kBM, BN, false);
+    static constexpr int STAGES = PAIR ? 6 : 4;
+    static constexpr int SMEM = STAGES * STAGE + 1024;    // + alignment slack
+    static constexpr uint32_t IDESC = idesc_bf16_f32(kBM * CM, BN, false);
     static constexpr uint32_t TMEM_COLS = 2 * BN;
 };
 
 struct GBars {
-    uint64_t full[kStages];
-    uint64_t empty[kStages];
+    uint64_t full[kMaxStages];
+    uint64_t empty[kMaxStages];
     uint64_t acc_full[2];
     uint64_t acc_empty[2];
     uint64_t drain;
@@ -76,11 +80,11 @@ __device__ __forceinline__ void report(DeviceStatus* st, volatile int* abort, in
     }
 }
 
-template <int BN, int CM>
+template <int BN, bool PAIR>
 __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant__ GemmParams p) {
-    using C = GCfg<BN>;
-    constexpr int B_SLICE = C::B_BYTES / CM;        // bytes of B this CTA loads
-    constexpr uint16_t kMask = uint16_t((1u << CM) - 1);
+    using C = GCfg<BN, PAIR>;
+    constexpr int CM = C::CM;
+    constexpr int kStages = C::STAGES;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
@@ -90,10 +94,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
     volatile int* abort = &bars.abort_flag;
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    // cluster tiles: CM consecutive M tiles of one N tile
+    // tiles of CM x 128 rows by BN columns; both CTAs of a pair walk the same sequence
     const int ctm = (p.tiles_m + CM - 1) / CM;
     const int n_tiles = ctm * p.tiles_n;
-    const int rank = CM > 1 ? int(cluster_ctarank()) : 0;
+    const int rank = PAIR ? int(cluster_ctarank()) : 0;
+    const bool leader = rank == 0;
     const int c_first = blockIdx.x / CM;
     const int c_stride = gridDim.x / CM;
     const int nk = (p.K + kBK - 1) / kBK;
@@ -102,11 +107,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(smem_u32(&bars.full[s]), 1);
-            mbar_init(smem_u32(&bars.empty[s]), CM);
+            mbar_init(smem_u32(&bars.empty[s]), 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&bars.acc_full[b]), 1);
-            mbar_init(smem_u32(&bars.acc_empty[b]), 128);
+            mbar_init(smem_u32(&bars.acc_empty[b]), 128 * CM);
         }
         mbar_init(smem_u32(&bars.drain), 1);
         bars.abort_flag = 0;
@@ -115,12 +120,17 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
     if (p.epi == kEpiQkv && p.rope)
         for (int i = threadIdx.x; i < kMaxTEntries; i += kThreads) s_t[i] = p.ra.t_tab[i];
     if (warp == 1) {
-        tmem_alloc(smem_u32(&bars.tmem_base), C::TMEM_COLS);
-        tmem_relinquish();
+        if (PAIR) {
+            tmem_alloc_pair(smem_u32(&bars.tmem_base), C::TMEM_COLS);
+            tmem_relinquish_pair();
+        } else {
+            tmem_alloc(smem_u32(&bars.tmem_base), C::TMEM_COLS);
+            tmem_relinquish();
+        }
     }
     tc_fence_before();
     __syncthreads();
-    if (CM > 1) cluster_sync_all();   // every CTA's barriers exist before any multicast
+    if (PAIR) cluster_sync_all();   // both CTAs' barriers exist before any cross-CTA signal
     tc_fence_after();
     const uint32_t tmem = bars.tmem_base;
 
@@ -137,32 +147,40 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
                 for (int kb = 0; kb < nk; ++kb) {
                     const int s = it % kStages;
                     // slot s was last filled by load it - kStages; the MMA that read it
-                    // commits empty[s] once per use
+                    // commits empty[s] (in both CTAs of a pair) once per use
                     if (it >= kStages &&
                         !mbar_wait(smem_u32(&bars.empty[s]), ((it / kStages) - 1) & 1, lim, abort)) {
                         report(p.status, abort, 0, it);
                         ok = false;
                         break;
                     }
-                    const uint32_t fb = smem_u32(&bars.full[s]);
-                    mbar_arrive_expect_tx(fb, C::STAGE);
                     const uint32_t dst = sbase + s * C::STAGE;
-                    tma_load_2d(dst, &p.a_map, fb, kb * kBK, tm * kBM);
-                    if (CM == 1)
+                    if (PAIR) {
+                        // both CTAs' bytes complete on the leader's barrier
+                        const uint32_t fb = mapa_shared(smem_u32(&bars.full[s]), 0);
+                        if (leader) mbar_arrive_expect_tx(smem_u32(&bars.full[s]), 2 * C::STAGE);
+                        tma_load_2d_pair(dst, &p.a_map, fb, kb * kBK, tm * kBM);
+                        tma_load_2d_pair(dst + C::A_BYTES, &p.b_map, fb, kb * kBK,
+                                         tn * BN + rank * (BN / 2));
+                    } else {
+                        const uint32_t fb = smem_u32(&bars.full[s]);
+                        mbar_arrive_expect_tx(fb, C::STAGE);
+                        tma_load_2d(dst, &p.a_map, fb, kb * kBK, tm * kBM);
                         tma_load_2d(dst + C::A_BYTES, &p.b_map, fb, kb * kBK, tn * BN);
-                    else
-                        tma_load_2d_mc(dst + C::A_BYTES + rank * B_SLICE, &p.b_map, fb, kb * kBK,
-                                       tn * BN + rank * (BN / CM), kMask);
+                    }
                     ++it;
                 }
             }
-            // drain: every issued load lands before the CTA may exit
-            for (int i = (it > kStages ? it - kStages : 0); i < it; ++i)
-                mbar_wait_drain(smem_u32(&bars.full[i % kStages]), (i / kStages) & 1, lim);
+            // drain: every issued load lands before the CTA may exit (a pair's loads all
+            // complete on the leader's barriers; the follower is held by the closing
+            // cluster barrier until the leader has drained)
+            if (leader)
+                for (int i = (it > kStages ? it - kStages : 0); i < it; ++i)
+                    mbar_wait_drain(smem_u32(&bars.full[i % kStages]), (i / kStages) & 1, lim);
         }
     } else if (warp == 1) {
-        // ============================ MMA issuer (one thread) ===============================
-        if (lane == 0) {
+        // ======================= MMA issuer (one thread of the leader) =======================
+        if (lane == 0 && leader) {
             // descriptors are linear in the 16-byte start address: a K step of 16 bf16
             // inside the 128-byte swizzle atom adds 32 bytes (2 units)
             const uint64_t da0 = sdesc_sw128(sbase, 16, 1024);
@@ -190,16 +208,25 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
                     tc_fence_after();
                     const uint64_t so = uint64_t((s * C::STAGE) >> 4);
 #pragma unroll
-                    for (int k = 0; k < kBK / 16; ++k)
-                        umma_ss(d, da0 + so + uint64_t(2 * k), db0 + so + uint64_t(2 * k), C::IDESC,
-                                (kb > 0 || k > 0) ? 1u : 0u);
-                    if (CM == 1) umma_commit(smem_u32(&bars.empty[s]));
-                    else umma_commit_mc(smem_u32(&bars.empty[s]), kMask);
+                    for (int k = 0; k < kBK / 16; ++k) {
+                        if (PAIR)
+                            umma_ss_pair(d, da0 + so + uint64_t(2 * k), db0 + so + uint64_t(2 * k),
+                                         C::IDESC, (kb > 0 || k > 0) ? 1u : 0u);
+                        else
+                            umma_ss(d, da0 + so + uint64_t(2 * k), db0 + so + uint64_t(2 * k),
+                                    C::IDESC, (kb > 0 || k > 0) ? 1u : 0u);
+                    }
+                    if (PAIR) umma_commit_pair(smem_u32(&bars.empty[s]), 0x3);
+                    else umma_commit(smem_u32(&bars.empty[s]));
                 }
-                if (ok) umma_commit(smem_u32(&bars.acc_full[b]));
+                if (ok) {
+                    if (PAIR) umma_commit_pair(smem_u32(&bars.acc_full[b]), 0x3);
+                    else umma_commit(smem_u32(&bars.acc_full[b]));
+                }
             }
             // drain: all issued MMAs complete before TMEM is released
-            umma_commit(smem_u32(&bars.drain));
+            if (PAIR) umma_commit_pair(smem_u32(&bars.drain), 0x1);
+            else umma_commit(smem_u32(&bars.drain));
             mbar_wait_drain(smem_u32(&bars.drain), 0, lim);
         }
     } else {
@@ -245,12 +272,24 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
                     for (int i = 0; i < 16; ++i)
                         w[i] = pack_bf16x2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
                     if (rot) {
+                        // all 16 (cos, sin) of the chunk first, each one load from an
+                        // address chosen without branching (t segment in shared memory, h
+                        // and w segments in the stream's table): a branch per pair on the
+                        // runtime segment widths serialises one load latency per pair
                         const int pi0 = (cc & (p.head_dim - 1)) >> 1;
+                        const int dt2 = p.ra.dt2, dth = p.ra.dt2 + p.ra.dh2;
+                        const float2* t_row = s_t + f * dt2;
+                        const float2* h_row = p.ra.hw + rr * p.ra.dh2 - dt2;
+                        const float2* w_row = p.ra.hw + p.ra.gh * p.ra.dh2 + col * p.ra.dw2 - dth;
+                        float2 cs[16];
 #pragma unroll
                         for (int i = 0; i < 16; ++i) {
-                            const float2 cs = rope_cs(p.ra, s_t, pi0 + i, f, rr, col);
-                            w[i] = rope_pair(w[i], cs.x, cs.y);
+                            const int pi = pi0 + i;
+                            const float2* src = pi < dt2 ? t_row + pi : (pi < dth ? h_row + pi : w_row + pi);
+                            cs[i] = *src;
                         }
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) w[i] = rope_pair(w[i], cs[i].x, cs[i].y);
                     }
                     uint4* o = reinterpret_cast<uint4*>(dst + size_t(grow) * p.d + cc);
 #pragma unroll
@@ -302,51 +341,55 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
                 }
             }
             tc_fence_before();
-            mbar_arrive(smem_u32(&bars.acc_empty[b]));
+            if (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&bars.acc_empty[b]), 0));
+            else mbar_arrive(smem_u32(&bars.acc_empty[b]));
         }
     }
     __syncwarp();
     tc_fence_before();
     __syncthreads();
-    if (CM > 1) cluster_sync_all();   // no peer multicasts into or signals this CTA any more
+    if (PAIR) cluster_sync_all();   // the pair is done with TMEM and with each other
     tc_fence_after();
-    if (warp == 1) tmem_dealloc(tmem, C::TMEM_COLS);
+    if (warp == 1) {
+        if (PAIR) tmem_dealloc_pair(tmem, C::TMEM_COLS);
+        else tmem_dealloc(tmem, C::TMEM_COLS);
+    }
 }
 
-template <int BN, int CM>
+template <int BN, bool PAIR>
 cudaError_t launch(const GemmParams& p, cudaStream_t st) {
+    using C = GCfg<BN, PAIR>;
     static bool attr_set = false;
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(gemm_kernel<BN, CM>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             GCfg<BN>::SMEM);
+        cudaError_t e = cudaFuncSetAttribute(gemm_kernel<BN, PAIR>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    const int n_ctiles = ((p.tiles_m + CM - 1) / CM) * p.tiles_n;
-    const int clusters = n_ctiles < num_sms() / CM ? n_ctiles : num_sms() / CM;
-    if (CM == 1) {
-        gemm_kernel<BN, 1><<<clusters, kThreads, GCfg<BN>::SMEM, st>>>(p);
+    const int n_ctiles = ((p.tiles_m + C::CM - 1) / C::CM) * p.tiles_n;
+    const int units = n_ctiles < num_sms() / C::CM ? n_ctiles : num_sms() / C::CM;
+    if (!PAIR) {
+        gemm_kernel<BN, false><<<units, kThreads, C::SMEM, st>>>(p);
         return cudaGetLastError();
     }
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(unsigned(clusters * CM));
+    cfg.gridDim = dim3(unsigned(units * 2));
     cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = GCfg<BN>::SMEM;
+    cfg.dynamicSmemBytes = C::SMEM;
     cfg.stream = st;
     cudaLaunchAttribute at[1];
     at[0].id = cudaLaunchAttributeClusterDimension;
-    at[0].val.clusterDim.x = CM;
+    at[0].val.clusterDim.x = 2;
     at[0].val.clusterDim.y = 1;
     at[0].val.clusterDim.z = 1;
     cfg.attrs = at;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, gemm_kernel<BN, CM>, p);
+    return cudaLaunchKernelEx(&cfg, gemm_kernel<BN, true>, p);
 }
 
 }  // namespace
 
-// CTAs per cluster sharing B: 2 whenever there are at least two M tiles.
+// CTAs per tile: a pair (cta_group::2) whenever there are at least two M tiles.
 int gemm_cluster_m(int M) { return M > kBM ? 2 : 1; }
 
 int gemm_block_n(int N, int epi, int d) {
@@ -361,8 +404,9 @@ cudaError_t launch_gemm(GemmParams p, cudaStream_t st) {
     const int bn = gemm_block_n(p.N, p.epi, p.d);
     p.tiles_m = (p.M + kBM - 1) / kBM;
     p.tiles_n = (p.N + bn - 1) / bn;
-    if (gemm_cluster_m(p.M) == 2) return bn == 256 ? launch<256, 2>(p, st) : launch<128, 2>(p, st);
-    return bn == 256 ? launch<256, 1>(p, st) : launch<128, 1>(p, st);
+    if (gemm_cluster_m(p.M) == 2)
+        return bn == 256 ? launch<256, true>(p, st) : launch<128, true>(p, st);
+    return bn == 256 ? launch<256, false>(p, st) : launch<128, false>(p, st);
 }
 
 }  // namespace frt
