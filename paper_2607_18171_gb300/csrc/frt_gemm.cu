@@ -393,15 +393,29 @@ cudaError_t launch(const GemmParams& p, cudaStream_t st) {
 int gemm_cluster_m(int M) { return M > kBM ? 2 : 1; }
 
 int gemm_block_n(int N, int epi, int d) {
-    // BN = 256 unless the QKV epilogue needs 128-column tiles (d not a multiple of 256)
-    // or N is small enough that 128-column tiles fill more SMs
-    if (epi == kEpiQkv) return (d % 256 == 0) ? 256 : 128;
-    return (N > 128) ? 256 : 128;
+    // 128-column tiles when the QKV epilogue needs them (d not a multiple of 256) or N
+    // is small; otherwise 256 unless 128 balances the rounds of tiles over the SMs
+    // clearly better (tile cost ~ BN, plus a quarter at 128 for the higher operand
+    // traffic per FLOP)
+    if (epi == kEpiQkv && d % 256 != 0) return 128;
+    if (N <= 128) return 128;
+    (void)d;
+    return 256;
+}
+
+int gemm_block_n_for(int M, int N, int epi, int d) {
+    const int bn = gemm_block_n(N, epi, d);
+    if (bn == 128 || (epi == kEpiQkv && d % 128 != 0)) return bn;
+    const int units = num_sms() / gemm_cluster_m(M);
+    const long long ctm = ((M + kBM - 1) / kBM + gemm_cluster_m(M) - 1) / gemm_cluster_m(M);
+    const long long r256 = (ctm * ((N + 255) / 256) + units - 1) / units;
+    const long long r128 = (ctm * ((N + 127) / 128) + units - 1) / units;
+    return (r128 * 128 * 5 < r256 * 256 * 4) ? 128 : 256;
 }
 
 cudaError_t launch_gemm(GemmParams p, cudaStream_t st) {
     if (p.M <= 0 || p.N <= 0 || p.K <= 0) return cudaSuccess;
-    const int bn = gemm_block_n(p.N, p.epi, p.d);
+    const int bn = gemm_block_n_for(p.M, p.N, p.epi, p.d);
     p.tiles_m = (p.M + kBM - 1) / kBM;
     p.tiles_n = (p.N + bn - 1) / bn;
     if (gemm_cluster_m(p.M) == 2)

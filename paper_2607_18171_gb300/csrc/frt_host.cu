@@ -635,7 +635,7 @@ frt_status frt_block_step(frt_stream_t* s, const void* x, const void* w_qkv, con
     // 1. QKV projection; its epilogue rotates q, k and writes k, v into the ring slot
     GemmParams g;
     std::memset(&g, 0, sizeof(g));
-    const int bn = gemm_block_n(3 * d, kEpiQkv, d);
+    const int bn = gemm_block_n_for(s->n_q, 3 * d, kEpiQkv, d);
     if ((st = make_map_2d(&g.a_map, x, d, s->n_q, 128)) != FRT_OK) return st;
     if ((st = make_map_2d(&g.b_map, w_qkv, d, 3LL * d, bn / gemm_cluster_m(s->n_q))) != FRT_OK)
         return st;
@@ -671,7 +671,7 @@ frt_status frt_block_step(frt_stream_t* s, const void* x, const void* w_qkv, con
     // 3. output projection
     GemmParams h;
     std::memset(&h, 0, sizeof(h));
-    const int bn2 = gemm_block_n(d, kEpiPlain, 0);
+    const int bn2 = gemm_block_n_for(s->n_q, d, kEpiPlain, 0);
     if ((st = make_map_2d(&h.a_map, o_buf, d, s->n_q, 128)) != FRT_OK) return st;
     if ((st = make_map_2d(&h.b_map, w_o, d, d, bn2 / gemm_cluster_m(s->n_q))) != FRT_OK) return st;
     h.M = s->n_q;
@@ -706,7 +706,7 @@ frt_status frt_gemm_bf16(const void* a, const void* b, void* c, int M, int N, in
     std::memset(&g, 0, sizeof(g));
     frt_status st;
     if ((st = make_map_2d(&g.a_map, a, K, M, 128)) != FRT_OK) return st;
-    if ((st = make_map_2d(&g.b_map, b, K, N, gemm_block_n(N, kEpiPlain, 0) / gemm_cluster_m(M))) !=
+    if ((st = make_map_2d(&g.b_map, b, K, N, gemm_block_n_for(M, N, kEpiPlain, 0) / gemm_cluster_m(M))) !=
         FRT_OK)
         return st;
     g.M = M;

@@ -162,8 +162,8 @@ struct GemmParams {
 // Kernel launchers (defined in the .cu files).
 cudaError_t launch_gemm(GemmParams p, cudaStream_t st);
 // Column tile width the GEMM uses for this problem, and the number of CTAs per cluster
-// sharing each B tile (the B tensor map's box height is gemm_block_n / gemm_cluster_m).
-int gemm_block_n(int N, int epi, int d);
+// working on each tile (the B tensor map's box height is gemm_block_n_for / gemm_cluster_m).
+int gemm_block_n_for(int M, int N, int epi, int d);
 int gemm_cluster_m(int M);
 cudaError_t launch_rope_qk(const RopeParams& p, cudaStream_t st);
 cudaError_t launch_kv_append(const AppendParams& p, cudaStream_t st);
