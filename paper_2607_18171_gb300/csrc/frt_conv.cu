@@ -18,7 +18,10 @@
 //   warp 1      TMEM allocator + single-thread tcgen05.mma issuer (M 128, N = BN, K 16);
 //   warps 2-5   epilogue (one thread per output pixel of the tile; bias added, pixels
 //               outside the frame not stored).
-// The accumulator is double-buffered in TMEM (2 x BN columns). A second, small kernel
+// The accumulator is double-buffered in TMEM (2 x BN columns). With enough tiles, two
+// CTAs of a cluster work as a pair on two pixel tiles with tcgen05.mma.cta_group::2 (M =
+// 256): each holds its own A and half of the weight tile, which cuts the bytes each SM
+// must take in per FLOP — what bounds this kernel. A second, small kernel
 // writes the next cache (last kt - 1 frames of (cache, chunk)) into the other half of a
 // ping-pong pair, so no launch reads what it writes.
 #include <algorithm>
@@ -38,7 +41,7 @@ constexpr int kBM = 128;         // output pixels per tile: 8 rows x 16 columns
 constexpr int kTileW = 16;
 constexpr int kTileH = 8;
 constexpr int kBK = 64;          // input channels per k-block (one 128-byte swizzle row)
-constexpr int kStages = 4;
+constexpr int kMaxStages = 6;
 constexpr int kTimeoutCode = 6;  // FRT_ERR_TIMEOUT
 constexpr int kMaxTaps = 64;
 
@@ -55,19 +58,21 @@ struct ConvParams {
     DeviceStatus* status;
 };
 
-template <int BN>
+template <int BN, bool PAIR>
 struct CCfg {
+    static constexpr int CM = PAIR ? 2 : 1;
     static constexpr int A_BYTES = kBM * kBK * 2;
-    static constexpr int B_BYTES = BN * kBK * 2;
+    static constexpr int B_BYTES = (BN / CM) * kBK * 2;
     static constexpr int STAGE = A_BYTES + B_BYTES;
-    static constexpr int SMEM = kStages * STAGE + 1024;
-    static constexpr uint32_t IDESC = idesc_bf16_f32(kBM, BN, false);
+    static constexpr int STAGES = PAIR ? 6 : 4;
+    static constexpr int SMEM = STAGES * STAGE + 1024;
+    static constexpr uint32_t IDESC = idesc_bf16_f32(kBM * CM, BN, false);
     static constexpr uint32_t TMEM_COLS = (2 * BN <= 256) ? 256 : 512;
 };
 
 struct CBars {
-    uint64_t full[kStages];
-    uint64_t empty[kStages];
+    uint64_t full[kMaxStages];
+    uint64_t empty[kMaxStages];
     uint64_t acc_full[2];
     uint64_t acc_empty[2];
     uint64_t drain;
@@ -90,20 +95,23 @@ __device__ __forceinline__ void report(DeviceStatus* st, volatile int* abort, in
 }
 
 // tile index -> (frame, tile row, tile column, N tile); N tiles vary fastest so CTAs
-// launched together share the input window
-__device__ __forceinline__ void tile_coords(const ConvParams& p, int t, int& f, int& th, int& tw,
-                                            int& tn) {
+// launched together share the input window. With pairs, tile t covers pixel tiles
+// 2 m and 2 m + 1 (one per CTA, `rank`) of the same N tile.
+__device__ __forceinline__ void tile_coords(const ConvParams& p, int t, int cm, int rank, int& f,
+                                            int& th, int& tw, int& tn) {
     tn = t % p.tiles_n;
-    int m = t / p.tiles_n;
+    int m = (t / p.tiles_n) * cm + rank;
     tw = m % p.tiles_w;
     m /= p.tiles_w;
     th = m % p.tiles_h;
     f = m / p.tiles_h;
 }
 
-template <int BN>
+template <int BN, bool PAIR>
 __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant__ ConvParams p) {
-    using C = CCfg<BN>;
+    using C = CCfg<BN, PAIR>;
+    constexpr int CM = C::CM;
+    constexpr int kStages = C::STAGES;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
@@ -116,6 +124,10 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     const int taps = p.kt * p.kh * p.kw;
     const int nk = taps * nkb;
     const uint64_t lim = p.wait_limit_ns;
+    const int rank = PAIR ? int(cluster_ctarank()) : 0;
+    const bool leader = rank == 0;
+    const int c_first = blockIdx.x / CM;
+    const int c_stride = gridDim.x / CM;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
@@ -124,18 +136,24 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&bars.acc_full[b]), 1);
-            mbar_init(smem_u32(&bars.acc_empty[b]), 128);
+            mbar_init(smem_u32(&bars.acc_empty[b]), 128 * CM);
         }
         mbar_init(smem_u32(&bars.drain), 1);
         bars.abort_flag = 0;
         fence_mbar_init();
     }
     if (warp == 1) {
-        tmem_alloc(smem_u32(&bars.tmem_base), C::TMEM_COLS);
-        tmem_relinquish();
+        if (PAIR) {
+            tmem_alloc_pair(smem_u32(&bars.tmem_base), C::TMEM_COLS);
+            tmem_relinquish_pair();
+        } else {
+            tmem_alloc(smem_u32(&bars.tmem_base), C::TMEM_COLS);
+            tmem_relinquish();
+        }
     }
     tc_fence_before();
     __syncthreads();
+    if (PAIR) cluster_sync_all();
     tc_fence_after();
     const uint32_t tmem = bars.tmem_base;
 
@@ -147,9 +165,9 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
             tma_prefetch_map(&p.w_map);
             int it = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < p.n_tiles && ok; t += gridDim.x) {
+            for (int t = c_first; t < p.n_tiles && ok; t += c_stride) {
                 int f, th, tw, tn;
-                tile_coords(p, t, f, th, tw, tn);
+                tile_coords(p, t, CM, rank, f, th, tw, tn);
                 for (int kk = 0; kk < nk; ++kk) {
                     const int s = it % kStages;
                     if (it >= kStages &&
@@ -165,31 +183,39 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
                     const int dh = rem / p.kw;
                     const int dw = rem - dh * p.kw;
                     const int src = f + dt - (p.kt - 1);      // frame of (cache, chunk) - cache
-                    const uint32_t fb = smem_u32(&bars.full[s]);
-                    mbar_arrive_expect_tx(fb, C::STAGE);
                     const uint32_t dst = sbase + s * C::STAGE;
                     const int cx = tw * kTileW + dw - p.kw / 2;
                     const int cy = th * kTileH + dh - p.kh / 2;
-                    if (src < 0)
-                        tma_load_4d(dst, &p.c_map, fb, kb * kBK, cx, cy, src + p.kt - 1);
-                    else
-                        tma_load_4d(dst, &p.x_map, fb, kb * kBK, cx, cy, src);
-                    tma_load_3d(dst + C::A_BYTES, &p.w_map, fb, kb * kBK, tn * BN, tap);
+                    const CUtensorMap* amap = src < 0 ? &p.c_map : &p.x_map;
+                    const int az = src < 0 ? src + p.kt - 1 : src;
+                    if (PAIR) {
+                        const uint32_t fb = mapa_shared(smem_u32(&bars.full[s]), 0);
+                        if (leader) mbar_arrive_expect_tx(smem_u32(&bars.full[s]), 2 * C::STAGE);
+                        tma_load_4d_pair(dst, amap, fb, kb * kBK, cx, cy, az);
+                        tma_load_3d_pair(dst + C::A_BYTES, &p.w_map, fb, kb * kBK,
+                                         tn * BN + rank * (BN / 2), tap);
+                    } else {
+                        const uint32_t fb = smem_u32(&bars.full[s]);
+                        mbar_arrive_expect_tx(fb, C::STAGE);
+                        tma_load_4d(dst, amap, fb, kb * kBK, cx, cy, az);
+                        tma_load_3d(dst + C::A_BYTES, &p.w_map, fb, kb * kBK, tn * BN, tap);
+                    }
                     ++it;
                 }
             }
-            for (int i = (it > kStages ? it - kStages : 0); i < it; ++i)
-                mbar_wait_drain(smem_u32(&bars.full[i % kStages]), (i / kStages) & 1, lim);
+            if (leader)
+                for (int i = (it > kStages ? it - kStages : 0); i < it; ++i)
+                    mbar_wait_drain(smem_u32(&bars.full[i % kStages]), (i / kStages) & 1, lim);
         }
     } else if (warp == 1) {
-        // ============================ MMA issuer (one thread) ===============================
-        if (lane == 0) {
+        // ======================= MMA issuer (one thread of the leader) =======================
+        if (lane == 0 && leader) {
             const uint64_t da0 = sdesc_sw128(sbase, 16, 1024);
             const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, 16, 1024);
             int it = 0;
             int tl = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < p.n_tiles && ok; t += gridDim.x, ++tl) {
+            for (int t = c_first; t < p.n_tiles && ok; t += c_stride, ++tl) {
                 const int b = tl & 1;
                 if (tl >= 2 &&
                     !mbar_wait(smem_u32(&bars.acc_empty[b]), ((tl >> 1) - 1) & 1, lim, abort)) {
@@ -209,14 +235,24 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
                     tc_fence_after();
                     const uint64_t so = uint64_t((s * C::STAGE) >> 4);
 #pragma unroll
-                    for (int k = 0; k < kBK / 16; ++k)
-                        umma_ss(d, da0 + so + uint64_t(2 * k), db0 + so + uint64_t(2 * k), C::IDESC,
-                                (kk > 0 || k > 0) ? 1u : 0u);
-                    umma_commit(smem_u32(&bars.empty[s]));
+                    for (int k = 0; k < kBK / 16; ++k) {
+                        if (PAIR)
+                            umma_ss_pair(d, da0 + so + uint64_t(2 * k), db0 + so + uint64_t(2 * k),
+                                         C::IDESC, (kk > 0 || k > 0) ? 1u : 0u);
+                        else
+                            umma_ss(d, da0 + so + uint64_t(2 * k), db0 + so + uint64_t(2 * k),
+                                    C::IDESC, (kk > 0 || k > 0) ? 1u : 0u);
+                    }
+                    if (PAIR) umma_commit_pair(smem_u32(&bars.empty[s]), 0x3);
+                    else umma_commit(smem_u32(&bars.empty[s]));
                 }
-                if (ok) umma_commit(smem_u32(&bars.acc_full[b]));
+                if (ok) {
+                    if (PAIR) umma_commit_pair(smem_u32(&bars.acc_full[b]), 0x3);
+                    else umma_commit(smem_u32(&bars.acc_full[b]));
+                }
             }
-            umma_commit(smem_u32(&bars.drain));
+            if (PAIR) umma_commit_pair(smem_u32(&bars.drain), 0x1);
+            else umma_commit(smem_u32(&bars.drain));
             mbar_wait_drain(smem_u32(&bars.drain), 0, lim);
         }
     } else {
@@ -225,10 +261,10 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
         const int row = sub * 32 + lane;                 // pixel of the tile: 16 per row
         const uint32_t lane_off = uint32_t(sub * 32) << 16;
         int tl = 0;
-        for (int t = blockIdx.x; t < p.n_tiles; t += gridDim.x, ++tl) {
+        for (int t = c_first; t < p.n_tiles; t += c_stride, ++tl) {
             const int b = tl & 1;
             int f, th, tw, tn;
-            tile_coords(p, t, f, th, tw, tn);
+            tile_coords(p, t, CM, rank, f, th, tw, tn);
             const bool got = mbar_wait(smem_u32(&bars.acc_full[b]), (tl >> 1) & 1, lim, abort);
             if (!__all_sync(0xffffffffu, got)) {
                 if (!got) report(p.status, abort, 2, tl);
@@ -237,7 +273,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
             tc_fence_after();
             const int h = th * kTileH + (row >> 4);
             const int w = tw * kTileW + (row & 15);
-            const bool live = h < p.H && w < p.W;
+            const bool live = f < p.F && h < p.H && w < p.W;
             const size_t obase = ((size_t(f) * p.H + h) * p.W + w) * p.cout + size_t(tn) * BN;
 #pragma unroll 1
             for (int c = 0; c < BN / 32; ++c) {
@@ -271,14 +307,19 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
                 __syncwarp();
             }
             tc_fence_before();
-            mbar_arrive(smem_u32(&bars.acc_empty[b]));
+            if (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&bars.acc_empty[b]), 0));
+            else mbar_arrive(smem_u32(&bars.acc_empty[b]));
         }
     }
     __syncwarp();
     tc_fence_before();
     __syncthreads();
+    if (PAIR) cluster_sync_all();
     tc_fence_after();
-    if (warp == 1) tmem_dealloc(tmem, C::TMEM_COLS);
+    if (warp == 1) {
+        if (PAIR) tmem_dealloc_pair(tmem, C::TMEM_COLS);
+        else tmem_dealloc(tmem, C::TMEM_COLS);
+    }
 }
 
 // next cache = last kt - 1 frames of (cache, chunk), written to the other ping-pong half
@@ -295,19 +336,34 @@ __global__ void cache_shift_kernel(const uint4* __restrict__ cache, const uint4*
     }
 }
 
-template <int BN>
+template <int BN, bool PAIR>
 cudaError_t launch_conv(ConvParams p, cudaStream_t st) {
+    using C = CCfg<BN, PAIR>;
     static bool attr = false;
     if (!attr) {
-        cudaError_t e = cudaFuncSetAttribute(conv_kernel<BN>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             CCfg<BN>::SMEM);
+        cudaError_t e = cudaFuncSetAttribute(conv_kernel<BN, PAIR>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
         if (e != cudaSuccess) return e;
         attr = true;
     }
-    const int grid = std::min(p.n_tiles, num_sms());
-    conv_kernel<BN><<<grid, kThreads, CCfg<BN>::SMEM, st>>>(p);
-    return cudaGetLastError();
+    const int units = std::min(p.n_tiles, num_sms() / C::CM);
+    if (!PAIR) {
+        conv_kernel<BN, false><<<units, kThreads, C::SMEM, st>>>(p);
+        return cudaGetLastError();
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(unsigned(units * 2));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = C::SMEM;
+    cfg.stream = st;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 2;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, conv_kernel<BN, true>, p);
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
@@ -345,21 +401,34 @@ bool encode(CUtensorMap* map, const void* base, int rank, const cuuint64_t* dims
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Output-channel tile: the widest of 256 / 192 / 128 / 64 dividing Cout that still gives
-// every SM a tile, else the one with the fewest waves.
-int choose_bn(int cout, long long m_tiles) {
+// Output-channel tile and pairing. Cost of one k-block on an SM ~ the larger of its MMA
+// time (BN / 2 cycles per 16-deep MMA, four of them) and the time to receive its operand
+// bytes at the ~40 bytes/cycle an SM takes in with all SMs loading (A 16 KB, plus its
+// share of the BN x 64 weight slice); every tile has the same number of k-blocks, and
+// tiles run in rounds over the SMs (or SM pairs), so the launch costs rounds x that.
+// The cheapest of the widths dividing Cout wins; pairs need at least two pixel tiles.
+int choose_bn(int cout, long long m_tiles, bool& pair) {
     const int cands[4] = {256, 192, 128, 64};
     const long long sms = num_sms();
     int best = 0;
     double best_t = 1e30;
-    for (int bn : cands) {
-        if (cout % bn) continue;
-        const long long tiles = m_tiles * (cout / bn);
-        const double waves = double((tiles + sms - 1) / sms);
-        const double t = waves * bn * (1.0 + 16.0 / bn);   // per-instruction overhead at small N
-        if (t < best_t - 1e-9) {
-            best_t = t;
-            best = bn;
+    for (int pr = 0; pr < 2; ++pr) {
+        if (pr == 1 && m_tiles < 2) continue;
+        const int cm = pr ? 2 : 1;
+        const long long units = sms / cm;
+        const long long mt = (m_tiles + cm - 1) / cm;
+        for (int bn : cands) {
+            if (cout % bn) continue;
+            const long long tiles = mt * (cout / bn);
+            const double rounds = double((tiles + units - 1) / units);
+            const double mma = 4.0 * bn / 2.0;
+            const double bytes = 16384.0 + double(bn / cm) * 128.0;
+            const double t = rounds * std::max(mma, bytes / 40.0);
+            if (t < best_t - 1e-9) {
+                best_t = t;
+                best = bn;
+                pair = pr == 1;
+            }
         }
     }
     return best;
@@ -478,11 +547,13 @@ frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w, const void
     p.tiles_w = (c->W + kTileW - 1) / kTileW;
     p.tiles_h = (c->H + kTileH - 1) / kTileH;
     const long long m_tiles = (long long)c->F * p.tiles_w * p.tiles_h;
-    const int bn = choose_bn(c->cout, m_tiles);
+    bool pair = false;
+    const int bn = choose_bn(c->cout, m_tiles, pair);
     if (bn == 0) return cfail(FRT_ERR_UNSUPPORTED, "Cout has no supported tile width");
     p.tiles_n = c->cout / bn;
-    if (m_tiles * p.tiles_n >= (1LL << 31)) return cfail(FRT_ERR_UNSUPPORTED, "too many tiles");
-    p.n_tiles = int(m_tiles * p.tiles_n);
+    const long long m_units = pair ? (m_tiles + 1) / 2 : m_tiles;
+    if (m_units * p.tiles_n >= (1LL << 31)) return cfail(FRT_ERR_UNSUPPORTED, "too many tiles");
+    p.n_tiles = int(m_units * p.tiles_n);
     const cuuint32_t abox[4] = {64, kTileW, kTileH, 1};
     const cuuint64_t xdims[4] = {cuuint64_t(c->cin), cuuint64_t(c->W), cuuint64_t(c->H),
                                  cuuint64_t(c->F)};
@@ -490,7 +561,7 @@ frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w, const void
                                  cuuint64_t(std::max(1, c->kt - 1))};
     const cuuint64_t wdims[3] = {cuuint64_t(c->cin), cuuint64_t(c->cout),
                                  cuuint64_t(c->kt * c->kh * c->kw)};
-    const cuuint32_t wbox[3] = {64, cuuint32_t(bn), 1};
+    const cuuint32_t wbox[3] = {64, cuuint32_t(pair ? bn / 2 : bn), 1};
     if (!encode(&p.x_map, x, 4, xdims, abox) || !encode(&p.c_map, c->cache[c->cur], 4, cdims, abox) ||
         !encode(&p.w_map, w, 3, wdims, wbox))
         return cfail(FRT_ERR_CUDA, "tensor map encoding failed");
@@ -500,11 +571,15 @@ frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w, const void
     p.wait_limit_ns = c->wait_limit_ns;
     p.status = c->status_dev;
     cudaError_t e;
-    switch (bn) {
-        case 256: e = launch_conv<256>(p, c->cs); break;
-        case 192: e = launch_conv<192>(p, c->cs); break;
-        case 128: e = launch_conv<128>(p, c->cs); break;
-        default: e = launch_conv<64>(p, c->cs); break;
+    switch (bn * 2 + (pair ? 1 : 0)) {
+        case 513: e = launch_conv<256, true>(p, c->cs); break;
+        case 512: e = launch_conv<256, false>(p, c->cs); break;
+        case 385: e = launch_conv<192, true>(p, c->cs); break;
+        case 384: e = launch_conv<192, false>(p, c->cs); break;
+        case 257: e = launch_conv<128, true>(p, c->cs); break;
+        case 256: e = launch_conv<128, false>(p, c->cs); break;
+        case 129: e = launch_conv<64, true>(p, c->cs); break;
+        default: e = launch_conv<64, false>(p, c->cs); break;
     }
     if (e != cudaSuccess) return cfail(FRT_ERR_CUDA, cudaGetErrorString(e));
     if (c->kt > 1) {
