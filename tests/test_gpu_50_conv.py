@@ -45,6 +45,9 @@ SMALL = {
     "conv_f1": synth.ConvWorkload("conv_f1", 24, 64, 256, 3, 3, 3, 9, 17, 1, 4),
     # no temporal taps: nothing cached
     "conv_kt1": synth.ConvWorkload("conv_kt1", 25, 64, 192, 1, 3, 3, 8, 16, 2, 2),
+    # an odd number of pixel tiles (3 frames x 1 tile): the last CTA pair has a second
+    # half past the chunk, which computes on zero-filled input and stores nothing
+    "conv_odd_tiles": synth.ConvWorkload("conv_odd_tiles", 26, 64, 128, 3, 3, 3, 5, 9, 3, 3),
 }
 
 
