@@ -189,6 +189,14 @@ frt_status frt_conv_configure(frt_conv_t* c, int out_dtype, void* cuda_stream);
  * (cache, x). Two launches (the convolution on the tensor cores, the cache update). */
 frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w,
                          const void* bias, void* y);
+/* Tile of the convolution kernel, for tuning and tests (no counterpart in the paper):
+ * bn = output channels per tile (64, 96, 128, 192 or 256, dividing Cout) and pair = 1
+ * for CTA pairs (tcgen05 cta_group::2, two pixel tiles per pair) or 0 for single
+ * CTAs; bn = 0 restores the automatic choice (a cost model of the launch). Applies
+ * to later frt_conv_step calls; results do not depend on it beyond fp32 rounding
+ * order, which is the same for every tile (each output sums its taps in one order).
+ * FRT_ERR_INVALID_ARG for other values. */
+frt_status frt_conv_set_tile(frt_conv_t* c, int bn, int pair);
 /* The current cache [kt-1, H, W, Cin] bf16 (device, read-only use). */
 frt_status frt_conv_cache(const frt_conv_t* c, const void** cache);
 /* Wait for the handle's work; returns FRT_ERR_TIMEOUT if a device wait gave up. */

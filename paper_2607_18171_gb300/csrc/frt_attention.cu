@@ -284,9 +284,10 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             int sv = 1 % C::STAGES, sk = 2 % C::STAGES;   // ring slots of V_j and K_{j+1}
             // An MMA issue returns only once the previous MMA has drained, so a blocking
             // wait at a group boundary idles the tensor pipe. P_g of the next PV group is
-            // therefore probed (non-blocking) from the shadow of the last MMAs of the
-            // group before it; when a probe has seen it complete, only the fence remains
-            // at the boundary.
+            // therefore probed (non-blocking) from the shadow of the last MMA of the group
+            // before it; when the probe has seen it complete, only the fence remains at
+            // the boundary. One probe, not several: a shared-memory access by this thread
+            // behind queued MMAs costs it ~140 cycles, more than an MMA's shadow.
             auto take_p = [&](int g, int j, bool seen) -> bool {
                 if (seen) {
                     tc_fence_after();
@@ -312,14 +313,14 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 });
                 if (!ok) break;
                 if (ng == 2) {
-                    if (more) issue_s(0, sk, [&](int k) { if (k >= 5 && !p1_seen) p1_seen = probe_p(1, j); });
+                    if (more) issue_s(0, sk, [&](int k) { if (k == D / 16 - 1) p1_seen = probe_p(1, j); });
                     else umma_commit(smem_u32(&bars->o_done[0]));
                     if (!(ok = take_p(1, j, p1_seen))) break;
                     p1_seen = false;
                     issue_o(1, sv, j > 0, nop);
                     if (more) issue_s(1, sk, [&](int k) {
                         if (k == 0) ok = wait_load(2 * j + 3);
-                        if (k >= 5 && !p0_seen) p0_seen = probe_p(0, j + 1);
+                        if (k == D / 16 - 1) p0_seen = probe_p(0, j + 1);
                     });
                     else umma_commit(smem_u32(&bars->o_done[1]));
                 } else {

@@ -9,21 +9,28 @@
 //         w[tap][o][c] * x_ext[t + dt][h + dh - kh/2][w + dw - kw/2][c]
 // with x_ext = (cache frames, chunk frames) and zero outside the frame.
 //
-// As an implicit GEMM: M = output pixels, N = Cout, K = taps x Cin. An M tile is 8 rows x
-// 16 columns of one output frame; for each tap the A tile is a TMA box of the input
-// frame (64 channels x 16 x 8) moved by the tap's offset: out-of-frame pixels arrive as
-// zeros, which is the spatial padding. The temporal tap picks the cache or the chunk
-// tensor map. B is the tap's [Cout, Cin] weight slice. Persistent kernel, 192 threads:
-//   warp 0      TMA producer (A box + B box per k-block of 64 channels, 4-stage ring);
+// As an implicit GEMM: M = output pixels, N = Cout, K = taps x Cin. An M tile is 16 rows
+// x 8 columns of one output frame. For each temporal tap and 64-channel block, ONE TMA
+// box brings in the tile's halo, (16 + kh - 1) x (8 + kw - 1) input pixels (out-of-frame
+// pixels arrive as zeros: the spatial padding), and all kh x kw spatial taps read their
+// A operand from it: the operand of tap (dh, dw) is the same 128-byte-swizzled halo seen
+// from a start address moved by (dh * halo_w + dw) pixel rows, with 8-row groups (one
+// tile row) halo_w * 128 bytes apart. tcgen05 applies the swizzle to absolute shared-
+// memory addresses, so any whole-row start is valid once the halo sits at a 1024-byte
+// boundary. This brings each input pixel into the SM about 1.4 times per temporal tap
+// and channel block instead of kh x kw times. B is the tap's [Cout, Cin] weight slice.
+// Persistent kernel, 224 threads:
+//   warp 0      TMA producer of the halo ring;
+//   warp 6      TMA producer of the weight ring (one slice per spatial tap);
 //   warp 1      TMEM allocator + single-thread tcgen05.mma issuer (M 128, N = BN, K 16);
 //   warps 2-5   epilogue (one thread per output pixel of the tile; bias added, pixels
 //               outside the frame not stored).
 // The accumulator is double-buffered in TMEM (2 x BN columns). With enough tiles, two
 // CTAs of a cluster work as a pair on two pixel tiles with tcgen05.mma.cta_group::2 (M =
-// 256): each holds its own A and half of the weight tile, which cuts the bytes each SM
-// must take in per FLOP — what bounds this kernel. A second, small kernel
-// writes the next cache (last kt - 1 frames of (cache, chunk)) into the other half of a
-// ping-pong pair, so no launch reads what it writes.
+// 256): each holds its own halo and half of the weight slice, which halves the weight
+// bytes each SM takes in per FLOP — with the halo, the larger share of what bounds this
+// kernel. A second, small kernel writes the next cache (last kt - 1 frames of (cache,
+// chunk)) into the other half of a ping-pong pair, so no launch reads what it writes.
 #include <algorithm>
 #include <cstring>
 #include <mutex>
@@ -36,24 +43,30 @@
 namespace frt {
 namespace {
 
-constexpr int kThreads = 192;
-constexpr int kBM = 128;         // output pixels per tile: 8 rows x 16 columns
-constexpr int kTileW = 16;
-constexpr int kTileH = 8;
+constexpr int kThreads = 224;
+constexpr int kBM = 128;         // output pixels per tile: 16 rows x 8 columns
+constexpr int kTileW = 8;        // one 8-row operand group = one tile row
+constexpr int kTileH = 16;
 constexpr int kBK = 64;          // input channels per k-block (one 128-byte swizzle row)
-constexpr int kMaxStages = 6;
+constexpr int kMaxStages = 8;
 constexpr int kTimeoutCode = 6;  // FRT_ERR_TIMEOUT
-constexpr int kMaxTaps = 64;
+constexpr int kSmemBudget = 225 * 1024;  // dynamic shared memory the two rings may take
 
 struct ConvParams {
-    CUtensorMap x_map;      // 4D (Cin, W, H, F) bf16 over the chunk, box (64, 16, 8, 1)
-    CUtensorMap c_map;      // 4D (Cin, W, H, kt - 1) over the cache (unused when kt == 1)
-    CUtensorMap w_map;      // 3D (Cin, Cout, taps) bf16 over the weights, box (64, BN, 1)
+    CUtensorMap x_map;      // 4D (Cin, W, H, F) bf16 over the chunk, box (64, halo_w, halo_h, 1)
+    CUtensorMap c_map;      // the same over the cache (unused when kt == 1)
+    CUtensorMap w_map;      // 3D (Cin, Cout, taps) bf16 over the weights, box (64, BN / pair, tb)
     const float* bias;      // [Cout]
     void* y;                // [F, H, W, Cout] fp32 or bf16
     int y_bf16;
     int cin, cout, kt, kh, kw, H, W, F;
     int tiles_w, tiles_h, tiles_n, n_tiles;
+    int halo_w, halo_h;     // 8 + kw - 1, 16 + kh - 1 input pixels
+    int halo_tx;            // bytes one halo box delivers: halo_w * halo_h * 128
+    int a_bytes;            // halo ring stage (halo_tx rounded up to 1024)
+    int a_stages, b_stages;
+    int tb;                 // spatial taps per weight-ring stage: kw (one kernel row) or 1
+    int b_stage;            // weight-ring stage bytes: tb * (BN / pair) * 128
     unsigned long long wait_limit_ns;
     DeviceStatus* status;
 };
@@ -61,18 +74,16 @@ struct ConvParams {
 template <int BN, bool PAIR>
 struct CCfg {
     static constexpr int CM = PAIR ? 2 : 1;
-    static constexpr int A_BYTES = kBM * kBK * 2;
     static constexpr int B_BYTES = (BN / CM) * kBK * 2;
-    static constexpr int STAGE = A_BYTES + B_BYTES;
-    static constexpr int STAGES = PAIR ? 6 : 4;
-    static constexpr int SMEM = STAGES * STAGE + 1024;
     static constexpr uint32_t IDESC = idesc_bf16_f32(kBM * CM, BN, false);
     static constexpr uint32_t TMEM_COLS = (2 * BN <= 256) ? 256 : 512;
 };
 
 struct CBars {
-    uint64_t full[kMaxStages];
-    uint64_t empty[kMaxStages];
+    uint64_t a_full[kMaxStages];
+    uint64_t a_empty[kMaxStages];
+    uint64_t b_full[kMaxStages];
+    uint64_t b_empty[kMaxStages];
     uint64_t acc_full[2];
     uint64_t acc_empty[2];
     uint64_t drain;
@@ -111,18 +122,19 @@ template <int BN, bool PAIR>
 __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant__ ConvParams p) {
     using C = CCfg<BN, PAIR>;
     constexpr int CM = C::CM;
-    constexpr int kStages = C::STAGES;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
     __shared__ CBars bars;
-    const uint32_t sbase = smem_u32(smem);
+    const uint32_t sA = smem_u32(smem);
+    const uint32_t sB = sA + uint32_t(p.a_stages * p.a_bytes);
     volatile int* abort = &bars.abort_flag;
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const int nkb = p.cin / kBK;
-    const int taps = p.kt * p.kh * p.kw;
-    const int nk = taps * nkb;
+    const int nhalo = p.kt * nkb;              // halos (k-block groups) per tile
+    const int sp = p.kh * p.kw;                // spatial taps per halo
+    const int ngrp = sp / p.tb;                // weight-ring stages per halo
     const uint64_t lim = p.wait_limit_ns;
     const int rank = PAIR ? int(cluster_ctarank()) : 0;
     const bool leader = rank == 0;
@@ -130,9 +142,13 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     const int c_stride = gridDim.x / CM;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kStages; ++s) {
-            mbar_init(smem_u32(&bars.full[s]), 1);
-            mbar_init(smem_u32(&bars.empty[s]), 1);
+        for (int s = 0; s < p.a_stages; ++s) {
+            mbar_init(smem_u32(&bars.a_full[s]), 1);
+            mbar_init(smem_u32(&bars.a_empty[s]), 1);
+        }
+        for (int s = 0; s < p.b_stages; ++s) {
+            mbar_init(smem_u32(&bars.b_full[s]), 1);
+            mbar_init(smem_u32(&bars.b_empty[s]), 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&bars.acc_full[b]), 1);
@@ -157,62 +173,115 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     tc_fence_after();
     const uint32_t tmem = bars.tmem_base;
 
+    // Every loop below keeps its ring slot and phase in counters that wrap, and advances
+    // coordinates and descriptors by additions: the single issuing threads must not spend
+    // the tensor pipe's time on integer divisions between MMAs or copies.
     if (warp == 0) {
-        // ==================================== TMA producer ===================================
+        // ================================ halo producer (TMA) ================================
         if (lane == 0) {
             tma_prefetch_map(&p.x_map);
             if (p.kt > 1) tma_prefetch_map(&p.c_map);
-            tma_prefetch_map(&p.w_map);
-            int it = 0;
+            int s = 0;
+            uint32_t ph = 0;
+            int ia = 0;
             bool ok = true;
             for (int t = c_first; t < p.n_tiles && ok; t += c_stride) {
                 int f, th, tw, tn;
                 tile_coords(p, t, CM, rank, f, th, tw, tn);
-                for (int kk = 0; kk < nk; ++kk) {
-                    const int s = it % kStages;
-                    if (it >= kStages &&
-                        !mbar_wait(smem_u32(&bars.empty[s]), ((it / kStages) - 1) & 1, lim, abort)) {
-                        report(p.status, abort, 0, it);
+                const int cx = tw * kTileW - p.kw / 2;
+                const int cy = th * kTileH - p.kh / 2;
+                int src = f - (p.kt - 1);                 // frame of (cache, chunk) - cache
+                int kb = 0;
+                for (int hi = 0; hi < nhalo; ++hi, ++ia) {
+                    if (ia >= p.a_stages && !mbar_test_wait(smem_u32(&bars.a_empty[s]), ph ^ 1) &&
+                        !mbar_wait(smem_u32(&bars.a_empty[s]), ph ^ 1, lim, abort)) {
+                        report(p.status, abort, 0, ia);
                         ok = false;
                         break;
                     }
-                    const int tap = kk / nkb;
-                    const int kb = kk - tap * nkb;
-                    const int dt = tap / (p.kh * p.kw);
-                    const int rem = tap - dt * p.kh * p.kw;
-                    const int dh = rem / p.kw;
-                    const int dw = rem - dh * p.kw;
-                    const int src = f + dt - (p.kt - 1);      // frame of (cache, chunk) - cache
-                    const uint32_t dst = sbase + s * C::STAGE;
-                    const int cx = tw * kTileW + dw - p.kw / 2;
-                    const int cy = th * kTileH + dh - p.kh / 2;
                     const CUtensorMap* amap = src < 0 ? &p.c_map : &p.x_map;
                     const int az = src < 0 ? src + p.kt - 1 : src;
+                    const uint32_t dst = sA + uint32_t(s * p.a_bytes);
                     if (PAIR) {
-                        const uint32_t fb = mapa_shared(smem_u32(&bars.full[s]), 0);
-                        if (leader) mbar_arrive_expect_tx(smem_u32(&bars.full[s]), 2 * C::STAGE);
-                        tma_load_4d_pair(dst, amap, fb, kb * kBK, cx, cy, az);
-                        tma_load_3d_pair(dst + C::A_BYTES, &p.w_map, fb, kb * kBK,
-                                         tn * BN + rank * (BN / 2), tap);
+                        if (leader) mbar_arrive_expect_tx(smem_u32(&bars.a_full[s]), 2 * p.halo_tx);
+                        tma_load_4d_pair(dst, amap, mapa_shared(smem_u32(&bars.a_full[s]), 0),
+                                         kb * kBK, cx, cy, az);
                     } else {
-                        const uint32_t fb = smem_u32(&bars.full[s]);
-                        mbar_arrive_expect_tx(fb, C::STAGE);
-                        tma_load_4d(dst, amap, fb, kb * kBK, cx, cy, az);
-                        tma_load_3d(dst + C::A_BYTES, &p.w_map, fb, kb * kBK, tn * BN, tap);
+                        mbar_arrive_expect_tx(smem_u32(&bars.a_full[s]), p.halo_tx);
+                        tma_load_4d(dst, amap, smem_u32(&bars.a_full[s]), kb * kBK, cx, cy, az);
                     }
-                    ++it;
+                    if (++s == p.a_stages) {
+                        s = 0;
+                        ph ^= 1;
+                    }
+                    if (++kb == nkb) {
+                        kb = 0;
+                        ++src;
+                    }
                 }
             }
             if (leader)
-                for (int i = (it > kStages ? it - kStages : 0); i < it; ++i)
-                    mbar_wait_drain(smem_u32(&bars.full[i % kStages]), (i / kStages) & 1, lim);
+                for (int i = (ia > p.a_stages ? ia - p.a_stages : 0); i < ia; ++i)
+                    mbar_wait_drain(smem_u32(&bars.a_full[i % p.a_stages]), (i / p.a_stages) & 1, lim);
+        }
+    } else if (warp == 6) {
+        // ================================ weight producer (TMA) ==============================
+        if (lane == 0) {
+            tma_prefetch_map(&p.w_map);
+            int s = 0;
+            uint32_t ph = 0;
+            int ib = 0;
+            bool ok = true;
+            for (int t = c_first; t < p.n_tiles && ok; t += c_stride) {
+                const int n0 = (t % p.tiles_n) * BN + rank * (BN / CM);
+                int kb = 0, tap0 = 0;                     // tap0 = first tap of this dt
+                for (int hi = 0; hi < nhalo && ok; ++hi) {
+                    for (int g = 0; g < ngrp; ++g, ++ib) {
+                        if (ib >= p.b_stages && !mbar_test_wait(smem_u32(&bars.b_empty[s]), ph ^ 1) &&
+                            !mbar_wait(smem_u32(&bars.b_empty[s]), ph ^ 1, lim, abort)) {
+                            report(p.status, abort, 3, ib);
+                            ok = false;
+                            break;
+                        }
+                        const uint32_t dst = sB + uint32_t(s * p.b_stage);
+                        const int tap = tap0 + g * p.tb;
+                        if (PAIR) {
+                            if (leader) mbar_arrive_expect_tx(smem_u32(&bars.b_full[s]), 2 * p.b_stage);
+                            tma_load_3d_pair(dst, &p.w_map, mapa_shared(smem_u32(&bars.b_full[s]), 0),
+                                             kb * kBK, n0, tap);
+                        } else {
+                            mbar_arrive_expect_tx(smem_u32(&bars.b_full[s]), p.b_stage);
+                            tma_load_3d(dst, &p.w_map, smem_u32(&bars.b_full[s]), kb * kBK, n0, tap);
+                        }
+                        if (++s == p.b_stages) {
+                            s = 0;
+                            ph ^= 1;
+                        }
+                    }
+                    if (++kb == nkb) {
+                        kb = 0;
+                        tap0 += sp;
+                    }
+                }
+            }
+            if (leader)
+                for (int i = (ib > p.b_stages ? ib - p.b_stages : 0); i < ib; ++i)
+                    mbar_wait_drain(smem_u32(&bars.b_full[i % p.b_stages]), (i / p.b_stages) & 1, lim);
         }
     } else if (warp == 1) {
         // ======================= MMA issuer (one thread of the leader) =======================
         if (lane == 0 && leader) {
-            const uint64_t da0 = sdesc_sw128(sbase, 16, 1024);
-            const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, 16, 1024);
-            int it = 0;
+            // descriptors are linear in the 16-byte start address (addresses stay below
+            // 256 KB, so the 14-bit field never carries): tap (dh, dw) of halo stage sa
+            // is da0 + sa * a_step + dh * halo_w * 8 + dw, k-step k adds 2 k
+            const uint64_t da0 = sdesc_sw128(sA, 16, uint32_t(p.halo_w * 128));
+            const uint64_t db0 = sdesc_sw128(sB, 16, 1024);
+            const uint32_t a_step = uint32_t(p.a_bytes >> 4);
+            const uint32_t row_skip = uint32_t((p.halo_w - p.kw) * 8);
+            const uint32_t b_step = uint32_t(p.b_stage >> 4);
+            int sa = 0, sb = 0;
+            uint32_t pa = 0, pb = 0;
+            int ia = 0, ib = 0;
             int tl = 0;
             bool ok = true;
             for (int t = c_first; t < p.n_tiles && ok; t += c_stride, ++tl) {
@@ -225,26 +294,55 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
                 }
                 tc_fence_after();
                 const uint32_t d = tmem + uint32_t(b * BN);
-                for (int kk = 0; kk < nk; ++kk, ++it) {
-                    const int s = it % kStages;
-                    if (!mbar_wait(smem_u32(&bars.full[s]), (it / kStages) & 1, lim, abort)) {
-                        report(p.status, abort, 1, it);
+                uint32_t accumulate = 0;
+                for (int hi = 0; hi < nhalo && ok; ++hi, ++ia) {
+                    if (!mbar_test_wait(smem_u32(&bars.a_full[sa]), pa) &&
+                        !mbar_wait(smem_u32(&bars.a_full[sa]), pa, lim, abort)) {
+                        report(p.status, abort, 1, ia);
                         ok = false;
                         break;
                     }
-                    tc_fence_after();
-                    const uint64_t so = uint64_t((s * C::STAGE) >> 4);
+                    uint64_t da = da0 + uint64_t(uint32_t(sa) * a_step);
+                    // a weight stage holds tb consecutive taps of one kernel row: one wait
+                    // per tb * 4 MMAs (a wait issued behind MMAs costs the issuing thread
+                    // ~200 cycles, which only a long enough MMA queue hides)
+                    for (int dh = 0; dh < p.kh && ok; ++dh, da += row_skip) {
+                        for (int dw = 0; dw < p.kw; dw += p.tb, ++ib) {
+                            if (!mbar_test_wait(smem_u32(&bars.b_full[sb]), pb) &&
+                                !mbar_wait(smem_u32(&bars.b_full[sb]), pb, lim, abort)) {
+                                report(p.status, abort, 4, ib);
+                                ok = false;
+                                break;
+                            }
+                            tc_fence_after();
+                            uint64_t db = db0 + uint64_t(uint32_t(sb) * b_step);
+                            for (int u = 0; u < p.tb; ++u, da += 8, db += uint64_t(C::B_BYTES >> 4)) {
 #pragma unroll
-                    for (int k = 0; k < kBK / 16; ++k) {
-                        if (PAIR)
-                            umma_ss_pair(d, da0 + so + uint64_t(2 * k), db0 + so + uint64_t(2 * k),
-                                         C::IDESC, (kk > 0 || k > 0) ? 1u : 0u);
-                        else
-                            umma_ss(d, da0 + so + uint64_t(2 * k), db0 + so + uint64_t(2 * k),
-                                    C::IDESC, (kk > 0 || k > 0) ? 1u : 0u);
+                                for (int k = 0; k < kBK / 16; ++k) {
+                                    if (PAIR)
+                                        umma_ss_pair(d, da + uint64_t(2 * k), db + uint64_t(2 * k),
+                                                     C::IDESC, accumulate);
+                                    else
+                                        umma_ss(d, da + uint64_t(2 * k), db + uint64_t(2 * k), C::IDESC,
+                                                accumulate);
+                                    accumulate = 1;
+                                }
+                            }
+                            if (PAIR) umma_commit_pair(smem_u32(&bars.b_empty[sb]), 0x3);
+                            else umma_commit(smem_u32(&bars.b_empty[sb]));
+                            if (++sb == p.b_stages) {
+                                sb = 0;
+                                pb ^= 1;
+                            }
+                        }
                     }
-                    if (PAIR) umma_commit_pair(smem_u32(&bars.empty[s]), 0x3);
-                    else umma_commit(smem_u32(&bars.empty[s]));
+                    if (!ok) break;
+                    if (PAIR) umma_commit_pair(smem_u32(&bars.a_empty[sa]), 0x3);
+                    else umma_commit(smem_u32(&bars.a_empty[sa]));
+                    if (++sa == p.a_stages) {
+                        sa = 0;
+                        pa ^= 1;
+                    }
                 }
                 if (ok) {
                     if (PAIR) umma_commit_pair(smem_u32(&bars.acc_full[b]), 0x3);
@@ -258,7 +356,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     } else {
         // ====================================== epilogue =====================================
         const int sub = warp & 3;
-        const int row = sub * 32 + lane;                 // pixel of the tile: 16 per row
+        const int row = sub * 32 + lane;                 // pixel of the tile: 8 per row
         const uint32_t lane_off = uint32_t(sub * 32) << 16;
         int tl = 0;
         for (int t = c_first; t < p.n_tiles; t += c_stride, ++tl) {
@@ -271,8 +369,8 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
                 break;
             }
             tc_fence_after();
-            const int h = th * kTileH + (row >> 4);
-            const int w = tw * kTileW + (row & 15);
+            const int h = th * kTileH + (row >> 3);
+            const int w = tw * kTileW + (row & 7);
             const bool live = f < p.F && h < p.H && w < p.W;
             const size_t obase = ((size_t(f) * p.H + h) * p.W + w) * p.cout + size_t(tn) * BN;
 #pragma unroll 1
@@ -339,22 +437,23 @@ __global__ void cache_shift_kernel(const uint4* __restrict__ cache, const uint4*
 template <int BN, bool PAIR>
 cudaError_t launch_conv(ConvParams p, cudaStream_t st) {
     using C = CCfg<BN, PAIR>;
-    static bool attr = false;
-    if (!attr) {
+    const int smem = p.a_stages * p.a_bytes + p.b_stages * p.b_stage + 1024;
+    static int attr = 0;
+    if (smem > attr) {
         cudaError_t e = cudaFuncSetAttribute(conv_kernel<BN, PAIR>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         if (e != cudaSuccess) return e;
-        attr = true;
+        attr = smem;
     }
     const int units = std::min(p.n_tiles, num_sms() / C::CM);
     if (!PAIR) {
-        conv_kernel<BN, false><<<units, kThreads, C::SMEM, st>>>(p);
+        conv_kernel<BN, false><<<units, kThreads, smem, st>>>(p);
         return cudaGetLastError();
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(unsigned(units * 2));
     cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = C::SMEM;
+    cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
     cudaLaunchAttribute at[1];
     at[0].id = cudaLaunchAttributeClusterDimension;
@@ -401,14 +500,36 @@ bool encode(CUtensorMap* map, const void* base, int rank, const cuuint64_t* dims
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Output-channel tile and pairing. Cost of one k-block on an SM ~ the larger of its MMA
-// time (BN / 2 cycles per 16-deep MMA, four of them) and the time to receive its operand
-// bytes at the ~40 bytes/cycle an SM takes in with all SMs loading (A 16 KB, plus its
-// share of the BN x 64 weight slice); every tile has the same number of k-blocks, and
-// tiles run in rounds over the SMs (or SM pairs), so the launch costs rounds x that.
-// The cheapest of the widths dividing Cout wins; pairs need at least two pixel tiles.
-int choose_bn(int cout, long long m_tiles, bool& pair) {
-    const int cands[4] = {256, 192, 128, 64};
+// Ring plan for one tile shape: a weight stage holds a whole kernel row of taps (tb = kw)
+// when three such stages fit beside the halo ring, else one tap; three halos in flight
+// when that leaves room for three weight stages, else two. Returns false if even two
+// halo and two weight stages do not fit.
+bool plan_rings(int a_bytes, int b_bytes, int kw, int& tb, int& a_stages, int& b_stages) {
+    const int room = kSmemBudget - 1024;
+    tb = 1;
+    a_stages = 2;
+    bool found = false;
+    for (int t : {kw, 1})
+        for (int as = 3; as >= 2 && !found; --as)
+            if (room - as * a_bytes >= 3 * t * b_bytes) {
+                tb = t;
+                a_stages = as;
+                found = true;
+            }
+    b_stages = std::min(kMaxStages, (room - a_stages * a_bytes) / (tb * b_bytes));
+    return b_stages >= 2;
+}
+
+// Output-channel tile and pairing, from a cost model measured on GB300 with this
+// kernel: a spatial tap costs its MMA issue time (four MMAs of max(BN / 2, 50) cycles,
+// 1.2x that for CTA pairs, whose MMAs issue slower) plus ~350 cycles of ring
+// bookkeeping (a shared-memory access by the issuing thread behind queued MMAs costs it
+// ~140 cycles), plus ~300 more when a weight stage holds a single tap; every tile has the
+// same number of taps and tiles run in rounds over the SMs (or SM pairs), so a launch
+// costs rounds x that. The cheapest of the widths dividing Cout wins; pairs need at
+// least two pixel tiles.
+int choose_bn(int cout, long long m_tiles, int a_bytes, int kw, bool& pair) {
+    const int cands[5] = {256, 192, 128, 96, 64};
     const long long sms = num_sms();
     int best = 0;
     double best_t = 1e30;
@@ -419,11 +540,12 @@ int choose_bn(int cout, long long m_tiles, bool& pair) {
         const long long mt = (m_tiles + cm - 1) / cm;
         for (int bn : cands) {
             if (cout % bn) continue;
+            int tb, as, bs;
+            if (!plan_rings(a_bytes, (bn / cm) * kBK * 2, kw, tb, as, bs)) continue;
             const long long tiles = mt * (cout / bn);
             const double rounds = double((tiles + units - 1) / units);
-            const double mma = 4.0 * bn / 2.0;
-            const double bytes = 16384.0 + double(bn / cm) * 128.0;
-            const double t = rounds * std::max(mma, bytes / 40.0);
+            const double mma = 4.0 * std::max(bn / 2.0, 50.0) * (pr ? 1.2 : 1.0);
+            const double t = rounds * (350.0 + mma + (tb == 1 && kw > 1 ? 300.0 : 0.0));
             if (t < best_t - 1e-9) {
                 best_t = t;
                 best = bn;
@@ -451,6 +573,8 @@ struct frt_conv {
     DeviceStatus* status_dev = nullptr;
     long long chunks = 0;
     unsigned long long wait_limit_ns = 2000000000ull;
+    int force_bn = 0;      // 0: the cost model picks the tile
+    int force_pair = 0;
 };
 
 namespace {
@@ -474,7 +598,7 @@ frt_conv_t* frt_conv_create(int cin, int cout, int kt, int kh, int kw, int grid_
                             int frames_per_chunk) {
     if (cin < 64 || cin % 64 || cout < 64 || cout % 64 || kt < 1 || kt > 4 || kh < 1 || kh > 7 ||
         kw < 1 || kw > 7 || kh % 2 == 0 || kw % 2 == 0 || grid_h < 1 || grid_w < 1 ||
-        frames_per_chunk < 1 || kt * kh * kw > kMaxTaps || (long long)grid_h * grid_w > (1LL << 24)) {
+        frames_per_chunk < 1 || (long long)grid_h * grid_w > (1LL << 24)) {
         set_last_error("need Cin, Cout multiples of 64, 1 <= kt <= 4, odd kh, kw <= 7, positive sizes");
         return nullptr;
     }
@@ -546,22 +670,31 @@ frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w, const void
     p.F = c->F;
     p.tiles_w = (c->W + kTileW - 1) / kTileW;
     p.tiles_h = (c->H + kTileH - 1) / kTileH;
+    p.halo_w = kTileW + c->kw - 1;
+    p.halo_h = kTileH + c->kh - 1;
+    p.halo_tx = p.halo_w * p.halo_h * kBK * 2;
+    p.a_bytes = (p.halo_tx + 1023) & ~1023;
     const long long m_tiles = (long long)c->F * p.tiles_w * p.tiles_h;
-    bool pair = false;
-    const int bn = choose_bn(c->cout, m_tiles, pair);
+    bool pair = c->force_pair != 0;
+    const int bn = c->force_bn != 0 ? c->force_bn
+                                    : choose_bn(c->cout, m_tiles, p.a_bytes, c->kw, pair);
     if (bn == 0) return cfail(FRT_ERR_UNSUPPORTED, "Cout has no supported tile width");
+    const int b_bytes = (pair ? bn / 2 : bn) * kBK * 2;
+    if (!plan_rings(p.a_bytes, b_bytes, c->kw, p.tb, p.a_stages, p.b_stages))
+        return cfail(FRT_ERR_UNSUPPORTED, "halo and weight rings do not fit");
+    p.b_stage = p.tb * b_bytes;
     p.tiles_n = c->cout / bn;
     const long long m_units = pair ? (m_tiles + 1) / 2 : m_tiles;
     if (m_units * p.tiles_n >= (1LL << 31)) return cfail(FRT_ERR_UNSUPPORTED, "too many tiles");
     p.n_tiles = int(m_units * p.tiles_n);
-    const cuuint32_t abox[4] = {64, kTileW, kTileH, 1};
+    const cuuint32_t abox[4] = {64, cuuint32_t(p.halo_w), cuuint32_t(p.halo_h), 1};
     const cuuint64_t xdims[4] = {cuuint64_t(c->cin), cuuint64_t(c->W), cuuint64_t(c->H),
                                  cuuint64_t(c->F)};
     const cuuint64_t cdims[4] = {cuuint64_t(c->cin), cuuint64_t(c->W), cuuint64_t(c->H),
                                  cuuint64_t(std::max(1, c->kt - 1))};
     const cuuint64_t wdims[3] = {cuuint64_t(c->cin), cuuint64_t(c->cout),
                                  cuuint64_t(c->kt * c->kh * c->kw)};
-    const cuuint32_t wbox[3] = {64, cuuint32_t(pair ? bn / 2 : bn), 1};
+    const cuuint32_t wbox[3] = {64, cuuint32_t(pair ? bn / 2 : bn), cuuint32_t(p.tb)};
     if (!encode(&p.x_map, x, 4, xdims, abox) || !encode(&p.c_map, c->cache[c->cur], 4, cdims, abox) ||
         !encode(&p.w_map, w, 3, wdims, wbox))
         return cfail(FRT_ERR_CUDA, "tensor map encoding failed");
@@ -578,6 +711,8 @@ frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w, const void
         case 384: e = launch_conv<192, false>(p, c->cs); break;
         case 257: e = launch_conv<128, true>(p, c->cs); break;
         case 256: e = launch_conv<128, false>(p, c->cs); break;
+        case 193: e = launch_conv<96, true>(p, c->cs); break;
+        case 192: e = launch_conv<96, false>(p, c->cs); break;
         case 129: e = launch_conv<64, true>(p, c->cs); break;
         default: e = launch_conv<64, false>(p, c->cs); break;
     }
@@ -596,6 +731,21 @@ frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w, const void
         c->cur ^= 1;
     }
     c->chunks += 1;
+    return FRT_OK;
+}
+
+frt_status frt_conv_set_tile(frt_conv_t* c, int bn, int pair) {
+    if (!c) return cfail(FRT_ERR_INVALID_ARG, "NULL conv handle");
+    if (bn == 0) {
+        c->force_bn = 0;
+        c->force_pair = 0;
+        return FRT_OK;
+    }
+    if ((bn != 64 && bn != 96 && bn != 128 && bn != 192 && bn != 256) || c->cout % bn != 0 ||
+        (pair != 0 && pair != 1))
+        return cfail(FRT_ERR_INVALID_ARG, "bn must be 64, 96, 128, 192 or 256 dividing Cout; pair 0 or 1");
+    c->force_bn = bn;
+    c->force_pair = pair;
     return FRT_OK;
 }
 

@@ -71,6 +71,7 @@ def lib() -> ctypes.CDLL:
         "frt_conv_configure": (I, [P, I, P]),
         "frt_conv_step": (I, [P, P, P, P, P]),
         "frt_conv_cache": (I, [P, ctypes.POINTER(P)]),
+        "frt_conv_set_tile": (I, [P, I, I]),
         "frt_conv_sync": (I, [P]),
         "frt_conv_reset": (I, [P]),
         "frt_conv_destroy": (None, [P]),
@@ -320,6 +321,10 @@ class ConvStream:
                 tuple(y.shape) != (self.frames, self.grid_h, self.grid_w, self.cout):
             raise ValueError("y must be a contiguous [F, H, W, Cout] CUDA tensor of the out dtype")
         _check(lib().frt_conv_step(self._h, _ptr(x), _ptr(w), _ptr(bias), _ptr(y)))
+
+    def set_tile(self, bn: int = 0, pair: int = 0) -> None:
+        """Force the kernel's output-channel tile and CTA pairing (bn = 0: automatic)."""
+        _check(lib().frt_conv_set_tile(self._h, bn, pair))
 
     def cache(self) -> torch.Tensor:
         p = ctypes.c_void_p()

@@ -1,7 +1,8 @@
 """GPU parity of the streaming causal 3D convolution (frt_conv_step) against the fp64
 oracle, through the C ABI: every output element at small sizes (ragged against the
-16 x 8 pixel tiles), sampled outputs at the VAE-decoder sizes, the frame cache
-bit-exact, determinism and the bf16 output.
+16-row x 8-column pixel tiles and their halos), every tile width and pairing the kernel
+offers, sampled outputs at the VAE-decoder sizes, the frame cache bit-exact,
+determinism and the bf16 output.
 
 Tolerance: fp32 accumulation of K = taps * Cin bf16 products, whatever the order, is
 within K * 2^-24 * sum |w x| of the exact sum (tested with K * 2^-23 plus 1e-6); a bf16
@@ -41,24 +42,32 @@ SMALL = {
     "convtiny": synth.CONV_WORKLOADS["convtiny"],
     # ragged against the tiles, kt = 2 and kh != kw, two k-blocks of channels
     "conv_ragged": synth.ConvWorkload("conv_ragged", 23, 128, 64, 2, 3, 5, 11, 21, 3, 3),
-    # one frame per chunk (the cache is shifted, not replaced), 256-wide N tiles
+    # one frame per chunk (the cache is shifted, not replaced)
     "conv_f1": synth.ConvWorkload("conv_f1", 24, 64, 256, 3, 3, 3, 9, 17, 1, 4),
     # no temporal taps: nothing cached
     "conv_kt1": synth.ConvWorkload("conv_kt1", 25, 64, 192, 1, 3, 3, 8, 16, 2, 2),
     # an odd number of pixel tiles (3 frames x 1 tile): the last CTA pair has a second
     # half past the chunk, which computes on zero-filled input and stores nothing
-    "conv_odd_tiles": synth.ConvWorkload("conv_odd_tiles", 26, 64, 128, 3, 3, 3, 5, 9, 3, 3),
+    "conv_odd_tiles": synth.ConvWorkload("conv_odd_tiles", 26, 64, 128, 3, 3, 3, 5, 7, 3, 3),
+    # a 7 x 7 spatial kernel (halo 14 x 22 pixels), two channel blocks
+    "conv_k7": synth.ConvWorkload("conv_k7", 27, 128, 64, 2, 7, 7, 19, 13, 2, 3),
 }
 
 
 @pytest.mark.parametrize("name", list(SMALL))
 @pytest.mark.parametrize("out", [torch.float32, torch.bfloat16])
 def test_conv_stream_matches_oracle_every_element(frt, name, out):
-    cw = SMALL[name]
+    _stream_against_oracle(frt, SMALL[name], name, out)
+
+
+def _stream_against_oracle(frt, cw, name, out, tile=None):
     w, b = synth.conv_weights(cw)
     wd, bd = w.cuda(), b.cuda()
     st = frt.ConvStream(cw.cin, cw.cout, cw.kt, cw.kh, cw.kw, cw.grid_h, cw.grid_w, cw.frames,
                         out_dtype=out)
+    if tile is not None:
+        st.set_tile(*tile)
+    outs = []
     orc = OracleConvStream(cw.cin, cw.cout, cw.kt, cw.kh, cw.kw, cw.grid_h, cw.grid_w)
     wf, bf = synth.as_f64(w), b.double().numpy()
     for c in range(cw.chunks):
@@ -69,12 +78,55 @@ def test_conv_stream_matches_oracle_every_element(frt, name, out):
         x_ext = np.concatenate([orc.cache, synth.as_f64(x)], axis=0)
         ref = orc.step(synth.as_f64(x), wf, bf)
         got = _f64(y)
+        outs.append(y)
         bound = _bound(cw, x_ext, wf, out == torch.bfloat16, ref)
         err = np.abs(got - ref)
         assert np.all(err <= bound), f"{name} chunk {c}: max excess {float(np.max(err - bound)):.3e}"
         if cw.kt > 1:
             assert np.array_equal(_f64(st.cache()), orc.cache), f"{name} chunk {c}: cache"
     st.close()
+    return outs
+
+
+# every output-channel tile and pairing the kernel offers, on shapes whose Cout admits
+# several of them (Cout 256: 64, 128, 256; Cout 192: 64, 96, 192)
+FORCED = [("conv_f1", bn, pr) for bn in (64, 128, 256) for pr in (0, 1)] + \
+         [("conv_kt1", bn, pr) for bn in (64, 96, 192) for pr in (0, 1)] + \
+         [("conv_odd_tiles", 128, 1), ("conv_ragged", 64, 0)]
+
+
+@pytest.mark.parametrize("name,bn,pair", FORCED)
+def test_conv_every_tile_matches_oracle(frt, name, bn, pair):
+    _stream_against_oracle(frt, SMALL[name], f"{name} bn={bn} pair={pair}", torch.float32,
+                           tile=(bn, pair))
+
+
+@pytest.mark.parametrize("name", ["conv_f1", "conv_kt1"])
+def test_conv_tile_choice_does_not_change_results(frt, name):
+    """Each output sums the same products in the same order (temporal tap, channel block,
+    spatial tap, 16-channel step) whatever the tile: every choice gives the same bits."""
+    cw = SMALL[name]
+    w, b = (t.cuda() for t in synth.conv_weights(cw))
+    results = {}
+    for bn in (64, 96, 128, 192, 256):
+        if cw.cout % bn:
+            continue
+        for pr in (0, 1):
+            st = frt.ConvStream(cw.cin, cw.cout, cw.kt, cw.kh, cw.kw, cw.grid_h, cw.grid_w,
+                                cw.frames)
+            st.set_tile(bn, pr)
+            ys = []
+            for c in range(cw.chunks):
+                y = st.new_out()
+                st.step(synth.conv_chunk(cw, 0, c).cuda(), w, b, y)
+                ys.append(y)
+            st.sync()
+            st.close()
+            results[(bn, pr)] = ys
+    first = next(iter(results.values()))
+    for key, ys in results.items():
+        for c, (a, r) in enumerate(zip(first, ys)):
+            assert torch.equal(a, r), f"{name}: tile {key} differs at chunk {c}"
 
 
 @pytest.mark.parametrize("name", ["vae30x52c384", "vae60x104c192"])
@@ -95,8 +147,8 @@ def test_conv_vae_sizes_on_sampled_pixels(frt, name):
         xf = synth.as_f64(x)
         x_ext = np.concatenate([cache, xf], axis=0)
         got = _f64(y)
-        pix = [(t, h, ww) for t in range(cw.frames) for h in (0, 7, 8, cw.grid_h - 1)
-               for ww in (0, 15, 16, cw.grid_w - 1)]
+        pix = [(t, h, ww) for t in range(cw.frames) for h in (0, 7, 8, 15, 16, cw.grid_h - 1)
+               for ww in (0, 7, 8, 15, 16, cw.grid_w - 1)]
         pix += [(int(rng.integers(cw.frames)), int(rng.integers(cw.grid_h)),
                  int(rng.integers(cw.grid_w))) for _ in range(300 - len(pix))]
         ph, pw = cw.kh // 2, cw.kw // 2
@@ -142,4 +194,7 @@ def test_conv_rejects_bad_arguments(frt):
     w, b = (t.cuda() for t in synth.conv_weights(cw))
     with pytest.raises(ValueError):
         st.step(torch.zeros(1, 2, 3, 64, dtype=torch.bfloat16, device="cuda"), w, b, st.new_out())
+    for bn, pr in ((100, 1), (128, 0), (64, 2)):    # not a width / not dividing Cout / pairing
+        with pytest.raises(frt.FrtError):
+            st.set_tile(bn, pr)
     st.close()
