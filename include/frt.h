@@ -193,8 +193,9 @@ frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w,
  * bn = output channels per tile (64, 96, 128, 192 or 256, dividing Cout) and pair = 1
  * for CTA pairs (tcgen05 cta_group::2, two pixel tiles per pair) or 0 for single
  * CTAs; bn = 0 restores the automatic choice (a cost model of the launch). Applies
- * to later frt_conv_step calls; results do not depend on it beyond fp32 rounding
- * order, which is the same for every tile (each output sums its taps in one order).
+ * to later frt_conv_step calls, which return FRT_ERR_UNSUPPORTED for bn = 96 with a
+ * bf16 output (staged in 64-channel units). Results do not depend on the tile: each
+ * output sums its products in one order (temporal tap, channel block, spatial tap).
  * FRT_ERR_INVALID_ARG for other values. */
 frt_status frt_conv_set_tile(frt_conv_t* c, int bn, int pair);
 /* The current cache [kt-1, H, W, Cin] bf16 (device, read-only use). */

@@ -23,8 +23,12 @@
 //   warp 0      TMA producer of the halo ring;
 //   warp 6      TMA producer of the weight ring (one slice per spatial tap);
 //   warp 1      TMEM allocator + single-thread tcgen05.mma issuer (M 128, N = BN, K 16);
-//   warps 2-5   epilogue (one thread per output pixel of the tile; bias added, pixels
-//               outside the frame not stored).
+//   warps 2-5   epilogue: one thread per output pixel of the tile adds the bias and
+//               writes its 128-byte slice of each column unit (32 fp32 or 64 bf16
+//               channels) into a 128-byte-swizzled staging slab, which one TMA tensor
+//               store writes to y (pixels outside the frame are clipped by the store);
+//               per-thread stores of whole pixel rows would touch 32 rows per warp
+//               instruction.
 // The accumulator is double-buffered in TMEM (2 x BN columns). With enough tiles, two
 // CTAs of a cluster work as a pair on two pixel tiles with tcgen05.mma.cta_group::2 (M =
 // 256): each holds its own halo and half of the weight slice, which halves the weight
@@ -50,12 +54,14 @@ constexpr int kTileH = 16;
 constexpr int kBK = 64;          // input channels per k-block (one 128-byte swizzle row)
 constexpr int kMaxStages = 8;
 constexpr int kTimeoutCode = 6;  // FRT_ERR_TIMEOUT
-constexpr int kSmemBudget = 225 * 1024;  // dynamic shared memory the two rings may take
+constexpr int kSmemBudget = 225 * 1024;  // dynamic shared memory of the kernel
+constexpr int kSlab = kBM * 128;         // epilogue staging: 128 rows of 128 bytes
 
 struct ConvParams {
     CUtensorMap x_map;      // 4D (Cin, W, H, F) bf16 over the chunk, box (64, halo_w, halo_h, 1)
     CUtensorMap c_map;      // the same over the cache (unused when kt == 1)
     CUtensorMap w_map;      // 3D (Cin, Cout, taps) bf16 over the weights, box (64, BN / pair, tb)
+    CUtensorMap y_map;      // 4D (Cout, W, H, F) fp32 or bf16 over y, box (32 | 64, 8, 16, 1)
     const float* bias;      // [Cout]
     void* y;                // [F, H, W, Cout] fp32 or bf16
     int y_bf16;
@@ -128,6 +134,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     __shared__ CBars bars;
     const uint32_t sA = smem_u32(smem);
     const uint32_t sB = sA + uint32_t(p.a_stages * p.a_bytes);
+    const uint32_t sStg = sB + uint32_t(p.b_stages * p.b_stage);   // 1024-aligned
     volatile int* abort = &bars.abort_flag;
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -358,28 +365,33 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
         const int sub = warp & 3;
         const int row = sub * 32 + lane;                 // pixel of the tile: 8 per row
         const uint32_t lane_off = uint32_t(sub * 32) << 16;
+        const uint32_t rb = sStg + uint32_t(row * 128);
+        const uint32_t sw = uint32_t(row & 7);
+        const bool est = threadIdx.x == 64;              // issues the tile's TMA stores
+        const int ucols = p.y_bf16 ? 64 : 32;            // output channels per unit
         int tl = 0;
         for (int t = c_first; t < p.n_tiles; t += c_stride, ++tl) {
             const int b = tl & 1;
             int f, th, tw, tn;
             tile_coords(p, t, CM, rank, f, th, tw, tn);
             const bool got = mbar_wait(smem_u32(&bars.acc_full[b]), (tl >> 1) & 1, lim, abort);
-            if (!__all_sync(0xffffffffu, got)) {
+            // all four warps go on or stop together: the staging below synchronises them
+            if (!named_bar_and(1, 128, got)) {
                 if (!got) report(p.status, abort, 2, tl);
                 break;
             }
             tc_fence_after();
-            const int h = th * kTileH + (row >> 3);
-            const int w = tw * kTileW + (row & 7);
-            const bool live = f < p.F && h < p.H && w < p.W;
-            const size_t obase = ((size_t(f) * p.H + h) * p.W + w) * p.cout + size_t(tn) * BN;
 #pragma unroll 1
-            for (int c = 0; c < BN / 32; ++c) {
-                uint32_t r[32];
-                tmem_ld32(tmem + lane_off + uint32_t(b * BN + c * 32), r);
-                tmem_ld_wait();
-                if (live) {
-                    const float4* bp = reinterpret_cast<const float4*>(p.bias + tn * BN + c * 32);
+            for (int u = 0; u < BN / ucols; ++u) {
+                if (est) bulk_wait_read<0>();            // the previous store has read the slab
+                named_bar_sync(1, 128);
+#pragma unroll 1
+                for (int h = 0; h < ucols / 32; ++h) {
+                    const int c = u * ucols + h * 32;    // first column of this TMEM load
+                    uint32_t r[32];
+                    tmem_ld32(tmem + lane_off + uint32_t(b * BN + c), r);
+                    tmem_ld_wait();
+                    const float4* bp = reinterpret_cast<const float4*>(p.bias + tn * BN + c);
                     float v[32];
 #pragma unroll
                     for (int i = 0; i < 8; ++i) {
@@ -390,24 +402,31 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
                         v[4 * i + 3] = __uint_as_float(r[4 * i + 3]) + bb.w;
                     }
                     if (p.y_bf16) {
-                        uint4* o = reinterpret_cast<uint4*>(static_cast<uint16_t*>(p.y) + obase + c * 32);
 #pragma unroll
                         for (int i = 0; i < 4; ++i)
-                            o[i] = make_uint4(pack_bf16x2(v[8 * i], v[8 * i + 1]), pack_bf16x2(v[8 * i + 2], v[8 * i + 3]),
-                                              pack_bf16x2(v[8 * i + 4], v[8 * i + 5]), pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
+                            st_shared_v4(rb + ((uint32_t(h * 4 + i) ^ sw) << 4),
+                                         pack_bf16x2(v[8 * i], v[8 * i + 1]), pack_bf16x2(v[8 * i + 2], v[8 * i + 3]),
+                                         pack_bf16x2(v[8 * i + 4], v[8 * i + 5]), pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
                     } else {
-                        float4* o = reinterpret_cast<float4*>(static_cast<float*>(p.y) + obase + c * 32);
 #pragma unroll
                         for (int i = 0; i < 8; ++i)
-                            o[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+                            st_shared_v4(rb + ((uint32_t(i) ^ sw) << 4), __float_as_uint(v[4 * i]),
+                                         __float_as_uint(v[4 * i + 1]), __float_as_uint(v[4 * i + 2]),
+                                         __float_as_uint(v[4 * i + 3]));
                     }
                 }
-                __syncwarp();
+                fence_proxy_async_smem();
+                named_bar_sync(1, 128);
+                if (est && f < p.F) {
+                    tma_store_4d(&p.y_map, sStg, tn * BN + u * ucols, tw * kTileW, th * kTileH, f);
+                    bulk_commit();
+                }
             }
             tc_fence_before();
             if (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&bars.acc_empty[b]), 0));
             else mbar_arrive(smem_u32(&bars.acc_empty[b]));
         }
+        if (est) bulk_wait<0>();                          // y written before the CTA exits
     }
     __syncwarp();
     tc_fence_before();
@@ -437,7 +456,7 @@ __global__ void cache_shift_kernel(const uint4* __restrict__ cache, const uint4*
 template <int BN, bool PAIR>
 cudaError_t launch_conv(ConvParams p, cudaStream_t st) {
     using C = CCfg<BN, PAIR>;
-    const int smem = p.a_stages * p.a_bytes + p.b_stages * p.b_stage + 1024;
+    const int smem = p.a_stages * p.a_bytes + p.b_stages * p.b_stage + kSlab + 1024;
     static int attr = 0;
     if (smem > attr) {
         cudaError_t e = cudaFuncSetAttribute(conv_kernel<BN, PAIR>,
@@ -485,19 +504,20 @@ EncodeTiledFn encode_fn() {
 }
 
 bool encode(CUtensorMap* map, const void* base, int rank, const cuuint64_t* dims,
-            const cuuint32_t* box) {
+            const cuuint32_t* box, bool f32 = false) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     cuuint64_t strides[3];
-    cuuint64_t acc = dims[0] * 2;
+    cuuint64_t acc = dims[0] * (f32 ? 4 : 2);
     for (int i = 0; i + 1 < rank; ++i) {
         strides[i] = acc;
         acc *= dims[i + 1];
     }
     cuuint32_t estr[4] = {1, 1, 1, 1};
-    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), dims, strides,
-              box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+    return fn(map, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank,
+              const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+              CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 // Ring plan for one tile shape: a weight stage holds a whole kernel row of taps (tb = kw)
@@ -505,7 +525,7 @@ bool encode(CUtensorMap* map, const void* base, int rank, const cuuint64_t* dims
 // when that leaves room for three weight stages, else two. Returns false if even two
 // halo and two weight stages do not fit.
 bool plan_rings(int a_bytes, int b_bytes, int kw, int& tb, int& a_stages, int& b_stages) {
-    const int room = kSmemBudget - 1024;
+    const int room = kSmemBudget - 1024 - kSlab;
     tb = 1;
     a_stages = 2;
     bool found = false;
@@ -527,8 +547,9 @@ bool plan_rings(int a_bytes, int b_bytes, int kw, int& tb, int& a_stages, int& b
 // ~140 cycles), plus ~300 more when a weight stage holds a single tap; every tile has the
 // same number of taps and tiles run in rounds over the SMs (or SM pairs), so a launch
 // costs rounds x that. The cheapest of the widths dividing Cout wins; pairs need at
-// least two pixel tiles.
-int choose_bn(int cout, long long m_tiles, int a_bytes, int kw, bool& pair) {
+// least two pixel tiles. A bf16 output is staged in 64-channel units, so its widths are
+// multiples of 64.
+int choose_bn(int cout, long long m_tiles, int a_bytes, int kw, bool y_bf16, bool& pair) {
     const int cands[5] = {256, 192, 128, 96, 64};
     const long long sms = num_sms();
     int best = 0;
@@ -539,7 +560,7 @@ int choose_bn(int cout, long long m_tiles, int a_bytes, int kw, bool& pair) {
         const long long units = sms / cm;
         const long long mt = (m_tiles + cm - 1) / cm;
         for (int bn : cands) {
-            if (cout % bn) continue;
+            if (cout % bn || (y_bf16 && bn % 64)) continue;
             int tb, as, bs;
             if (!plan_rings(a_bytes, (bn / cm) * kBK * 2, kw, tb, as, bs)) continue;
             const long long tiles = mt * (cout / bn);
@@ -676,9 +697,12 @@ frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w, const void
     p.a_bytes = (p.halo_tx + 1023) & ~1023;
     const long long m_tiles = (long long)c->F * p.tiles_w * p.tiles_h;
     bool pair = c->force_pair != 0;
+    const bool y_bf16 = c->out_dtype == FRT_OUT_BF16;
     const int bn = c->force_bn != 0 ? c->force_bn
-                                    : choose_bn(c->cout, m_tiles, p.a_bytes, c->kw, pair);
+                                    : choose_bn(c->cout, m_tiles, p.a_bytes, c->kw, y_bf16, pair);
     if (bn == 0) return cfail(FRT_ERR_UNSUPPORTED, "Cout has no supported tile width");
+    if (y_bf16 && bn % 64)
+        return cfail(FRT_ERR_UNSUPPORTED, "a bf16 output needs a tile width that is a multiple of 64");
     const int b_bytes = (pair ? bn / 2 : bn) * kBK * 2;
     if (!plan_rings(p.a_bytes, b_bytes, c->kw, p.tb, p.a_stages, p.b_stages))
         return cfail(FRT_ERR_UNSUPPORTED, "halo and weight rings do not fit");
@@ -695,8 +719,12 @@ frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w, const void
     const cuuint64_t wdims[3] = {cuuint64_t(c->cin), cuuint64_t(c->cout),
                                  cuuint64_t(c->kt * c->kh * c->kw)};
     const cuuint32_t wbox[3] = {64, cuuint32_t(pair ? bn / 2 : bn), cuuint32_t(p.tb)};
+    const bool y_f32 = c->out_dtype != FRT_OUT_BF16;
+    const cuuint64_t ydims[4] = {cuuint64_t(c->cout), cuuint64_t(c->W), cuuint64_t(c->H),
+                                 cuuint64_t(c->F)};
+    const cuuint32_t ybox[4] = {y_f32 ? 32u : 64u, kTileW, kTileH, 1};
     if (!encode(&p.x_map, x, 4, xdims, abox) || !encode(&p.c_map, c->cache[c->cur], 4, cdims, abox) ||
-        !encode(&p.w_map, w, 3, wdims, wbox))
+        !encode(&p.w_map, w, 3, wdims, wbox) || !encode(&p.y_map, y, 4, ydims, ybox, y_f32))
         return cfail(FRT_ERR_CUDA, "tensor map encoding failed");
     p.bias = static_cast<const float*>(bias);
     p.y = y;

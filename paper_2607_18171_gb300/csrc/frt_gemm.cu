@@ -3,12 +3,20 @@
 // DiT block (QKV projection in front of it, output projection after it).
 //
 // Persistent kernel, one CTA per SM, 192 threads:
-//   warp 0      TMA producer: A (128 x 64) and B (BN x 64) k-blocks, 128-byte swizzle,
-//               through a kStages-deep shared-memory ring;
+//   warp 0      TMA producer: two k-blocks of A (128 x 64 each) and of B (BN x 64 each)
+//               per ring stage, 128-byte swizzle, through a shared-memory ring (with K a
+//               multiple of 64, one box per operand loads both k-blocks through a 3D view
+//               (64, rows, K / 64) of the matrix);
 //   warp 1      TMEM allocator + single-thread tcgen05.mma issuer (M = 128, N = BN, K = 16
-//               per instruction, four per k-block);
+//               per instruction, eight per stage: one barrier wait per eight MMAs, since a
+//               shared-memory access by the issuing thread behind queued MMAs stalls it
+//               ~140 cycles);
 //   warps 2-5   epilogue: one thread per accumulator row (TMEM lane), 32 columns per
-//               tcgen05.ld.
+//               tcgen05.ld; each 128-byte column unit of the tile (32 fp32 or 64 bf16
+//               columns) is staged in a 128-byte-swizzled shared-memory slab and written
+//               by one TMA tensor store (rows past M and columns past N are clipped by
+//               the store); per-thread row stores would touch 32 rows per warp
+//               instruction.
 // The accumulator is double-buffered in TMEM (2 x BN columns), so the epilogue of tile i
 // runs while the tensor pipe computes tile i + 1.
 // When M spans more than one 128-row tile, two CTAs of a cluster work as a pair on a
@@ -42,16 +50,19 @@ constexpr int kThreads = 192;
 constexpr int kBM = 128;
 constexpr int kBK = 64;          // one 128-byte swizzle atom of bf16
 constexpr int kMaxStages = 6;
+constexpr int kKPS = 2;          // k-blocks per ring stage
 constexpr int kTimeoutCode = 6;  // FRT_ERR_TIMEOUT
 
 template <int BN, bool PAIR>
 struct GCfg {
     static constexpr int CM = PAIR ? 2 : 1;               // CTAs per tile
-    static constexpr int A_BYTES = kBM * kBK * 2;         // this CTA's 128 rows of A
-    static constexpr int B_BYTES = (BN / CM) * kBK * 2;   // this CTA's share of B
-    static constexpr int STAGE = A_BYTES + B_BYTES;
-    static constexpr int STAGES = PAIR ? 6 : 4;
-    static constexpr int SMEM = STAGES * STAGE + 1024;    // + alignment slack
+    static constexpr int A_BYTES = kBM * kBK * 2;         // this CTA's 128 rows of A, one k-block
+    static constexpr int B_BYTES = (BN / CM) * kBK * 2;   // this CTA's share of B, one k-block
+    static constexpr int STAGE = kKPS * (A_BYTES + B_BYTES);   // [A kb0 | A kb1 | B kb0 | B kb1]
+    static constexpr int SLAB = kBM * 128;                // epilogue staging slab
+    static constexpr int STAGES = (225 * 1024 - 1024 - SLAB) / STAGE < kMaxStages
+                                      ? (225 * 1024 - 1024 - SLAB) / STAGE : kMaxStages;
+    static constexpr int SMEM = STAGES * STAGE + SLAB + 1024;   // + alignment slack
     static constexpr uint32_t IDESC = idesc_bf16_f32(kBM * CM, BN, false);
     static constexpr uint32_t TMEM_COLS = 2 * BN;
 };
@@ -144,29 +155,46 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
             for (int t = c_first; t < n_tiles && ok; t += c_stride) {
                 const int tm = (t % ctm) * CM + rank;
                 const int tn = t / ctm;
-                for (int kb = 0; kb < nk; ++kb) {
+                const int brow = tn * BN + rank * (BN / CM);
+                for (int kb = 0; kb < nk; kb += kKPS) {
                     const int s = it % kStages;
                     // slot s was last filled by load it - kStages; the MMA that read it
                     // commits empty[s] (in both CTAs of a pair) once per use
-                    if (it >= kStages &&
+                    if (it >= kStages && !mbar_test_wait(smem_u32(&bars.empty[s]), ((it / kStages) - 1) & 1) &&
                         !mbar_wait(smem_u32(&bars.empty[s]), ((it / kStages) - 1) & 1, lim, abort)) {
                         report(p.status, abort, 0, it);
                         ok = false;
                         break;
                     }
                     const uint32_t dst = sbase + s * C::STAGE;
+                    const uint32_t dst_b = dst + kKPS * C::A_BYTES;
+                    // both k-blocks of the stage; past K (or past the last k-block) the
+                    // copies read zeros, and the bytes still count
                     if (PAIR) {
                         // both CTAs' bytes complete on the leader's barrier
                         const uint32_t fb = mapa_shared(smem_u32(&bars.full[s]), 0);
                         if (leader) mbar_arrive_expect_tx(smem_u32(&bars.full[s]), 2 * C::STAGE);
-                        tma_load_2d_pair(dst, &p.a_map, fb, kb * kBK, tm * kBM);
-                        tma_load_2d_pair(dst + C::A_BYTES, &p.b_map, fb, kb * kBK,
-                                         tn * BN + rank * (BN / 2));
+                        if (p.kview3) {
+                            tma_load_3d_pair(dst, &p.a_map, fb, 0, tm * kBM, kb);
+                            tma_load_3d_pair(dst_b, &p.b_map, fb, 0, brow, kb);
+                        } else {
+                            for (int h = 0; h < kKPS; ++h) {
+                                tma_load_2d_pair(dst + h * C::A_BYTES, &p.a_map, fb, (kb + h) * kBK, tm * kBM);
+                                tma_load_2d_pair(dst_b + h * C::B_BYTES, &p.b_map, fb, (kb + h) * kBK, brow);
+                            }
+                        }
                     } else {
                         const uint32_t fb = smem_u32(&bars.full[s]);
                         mbar_arrive_expect_tx(fb, C::STAGE);
-                        tma_load_2d(dst, &p.a_map, fb, kb * kBK, tm * kBM);
-                        tma_load_2d(dst + C::A_BYTES, &p.b_map, fb, kb * kBK, tn * BN);
+                        if (p.kview3) {
+                            tma_load_3d(dst, &p.a_map, fb, 0, tm * kBM, kb);
+                            tma_load_3d(dst_b, &p.b_map, fb, 0, brow, kb);
+                        } else {
+                            for (int h = 0; h < kKPS; ++h) {
+                                tma_load_2d(dst + h * C::A_BYTES, &p.a_map, fb, (kb + h) * kBK, tm * kBM);
+                                tma_load_2d(dst_b + h * C::B_BYTES, &p.b_map, fb, (kb + h) * kBK, brow);
+                            }
+                        }
                     }
                     ++it;
                 }
@@ -184,7 +212,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
             // descriptors are linear in the 16-byte start address: a K step of 16 bf16
             // inside the 128-byte swizzle atom adds 32 bytes (2 units)
             const uint64_t da0 = sdesc_sw128(sbase, 16, 1024);
-            const uint64_t db0 = sdesc_sw128(sbase + C::A_BYTES, 16, 1024);
+            const uint64_t db0 = sdesc_sw128(sbase + kKPS * C::A_BYTES, 16, 1024);
             int it = 0;
             int tl = 0;
             bool ok = true;
@@ -198,9 +226,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
                 }
                 tc_fence_after();
                 const uint32_t d = tmem + uint32_t(b * BN);
-                for (int kb = 0; kb < nk; ++kb, ++it) {
+                for (int kb = 0; kb < nk; kb += kKPS, ++it) {
                     const int s = it % kStages;
-                    if (!mbar_wait(smem_u32(&bars.full[s]), (it / kStages) & 1, lim, abort)) {
+                    if (!mbar_test_wait(smem_u32(&bars.full[s]), (it / kStages) & 1) &&
+                        !mbar_wait(smem_u32(&bars.full[s]), (it / kStages) & 1, lim, abort)) {
                         report(p.status, abort, 1, it);
                         ok = false;
                         break;
@@ -208,13 +237,18 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
                     tc_fence_after();
                     const uint64_t so = uint64_t((s * C::STAGE) >> 4);
 #pragma unroll
-                    for (int k = 0; k < kBK / 16; ++k) {
-                        if (PAIR)
-                            umma_ss_pair(d, da0 + so + uint64_t(2 * k), db0 + so + uint64_t(2 * k),
-                                         C::IDESC, (kb > 0 || k > 0) ? 1u : 0u);
-                        else
-                            umma_ss(d, da0 + so + uint64_t(2 * k), db0 + so + uint64_t(2 * k),
-                                    C::IDESC, (kb > 0 || k > 0) ? 1u : 0u);
+                    for (int h = 0; h < kKPS; ++h) {
+                        if (kb + h >= nk) break;          // the zero-filled half of the last stage
+                        const uint64_t da = da0 + so + uint64_t((h * C::A_BYTES) >> 4);
+                        const uint64_t db = db0 + so + uint64_t((h * C::B_BYTES) >> 4);
+#pragma unroll
+                        for (int k = 0; k < kBK / 16; ++k) {
+                            const uint32_t acc = (kb + h > 0 || k > 0) ? 1u : 0u;
+                            if (PAIR)
+                                umma_ss_pair(d, da + uint64_t(2 * k), db + uint64_t(2 * k), C::IDESC, acc);
+                            else
+                                umma_ss(d, da + uint64_t(2 * k), db + uint64_t(2 * k), C::IDESC, acc);
+                        }
                     }
                     if (PAIR) umma_commit_pair(smem_u32(&bars.empty[s]), 0x3);
                     else umma_commit(smem_u32(&bars.empty[s]));
@@ -234,13 +268,31 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
         const int sub = warp & 3;                      // TMEM lane quarter of this warp
         const int row = sub * 32 + lane;
         const uint32_t lane_off = uint32_t(sub * 32) << 16;
+        const uint32_t stg = sbase + uint32_t(kStages * C::STAGE);   // 1024-aligned slab
+        const uint32_t rb = stg + uint32_t(row * 128);
+        const uint32_t sw = uint32_t(row & 7);
+        const bool est = threadIdx.x == 64;            // issues the TMA stores
+        // slab free (the previous store has read it), then every thread refills it
+        auto slab_acquire = [&]() {
+            if (est) bulk_wait_read<0>();
+            named_bar_sync(1, 128);
+        };
+        auto slab_release = [&](const CUtensorMap* map, int c0, int r0) {
+            fence_proxy_async_smem();
+            named_bar_sync(1, 128);
+            if (est) {
+                tma_store_2d(map, stg, c0, r0);
+                bulk_commit();
+            }
+        };
         int tl = 0;
         for (int t = c_first; t < n_tiles; t += c_stride, ++tl) {
             const int b = tl & 1;
             const int tm = (t % ctm) * CM + rank;
             const int tn = t / ctm;
             const bool got = mbar_wait(smem_u32(&bars.acc_full[b]), (tl >> 1) & 1, lim, abort);
-            if (!__all_sync(0xffffffffu, got)) {
+            // all four warps go on or stop together: the staging below synchronises them
+            if (!named_bar_and(1, 128, got)) {
                 if (!got) report(p.status, abort, 2, tl);
                 break;
             }
@@ -251,8 +303,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
             if (p.epi == kEpiQkv) {
                 const int which = n0 / p.d;                 // 0 q, 1 k, 2 v
                 const int cbase = n0 - which * p.d;
-                uint16_t* dst = which == 0 ? p.q_out : (which == 1 ? p.k_out : p.v_out);
-                const bool rot = p.rope && which < 2;
+                const bool rot = p.rope && which < 2 && live;
                 int f = 0, rr = 0, col = 0;
                 if (rot) {
                     f = grow / p.ra.tpf;
@@ -261,89 +312,80 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
                     col = rem - rr * p.ra.gw;
                 }
 #pragma unroll 1
-                for (int c = 0; c < BN / 32; ++c) {
-                    uint32_t r[32];
-                    tmem_ld32(tmem + lane_off + uint32_t(b * BN + c * 32), r);
-                    tmem_ld_wait();
-                    if (live) {
-                    const int cc = cbase + c * 32;
-                    uint32_t w[16];
+                for (int u = 0; u < BN / 64; ++u) {      // 64 bf16 columns per unit
+                    slab_acquire();
+#pragma unroll 1
+                    for (int hh = 0; hh < 2; ++hh) {
+                        const int c = 2 * u + hh;
+                        uint32_t r[32];
+                        tmem_ld32(tmem + lane_off + uint32_t(b * BN + c * 32), r);
+                        tmem_ld_wait();
+                        const int cc = cbase + c * 32;
+                        uint32_t w[16];
 #pragma unroll
-                    for (int i = 0; i < 16; ++i)
-                        w[i] = pack_bf16x2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
-                    if (rot) {
-                        // all 16 (cos, sin) of the chunk first, each one load from an
-                        // address chosen without branching (t segment in shared memory, h
-                        // and w segments in the stream's table): a branch per pair on the
-                        // runtime segment widths serialises one load latency per pair
-                        const int pi0 = (cc & (p.head_dim - 1)) >> 1;
-                        const int dt2 = p.ra.dt2, dth = p.ra.dt2 + p.ra.dh2;
-                        const float2* t_row = s_t + f * dt2;
-                        const float2* h_row = p.ra.hw + rr * p.ra.dh2 - dt2;
-                        const float2* w_row = p.ra.hw + p.ra.gh * p.ra.dh2 + col * p.ra.dw2 - dth;
-                        float2 cs[16];
+                        for (int i = 0; i < 16; ++i)
+                            w[i] = pack_bf16x2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
+                        if (rot) {
+                            // all 16 (cos, sin) of the chunk first, each one load from an
+                            // address chosen without branching (t segment in shared memory,
+                            // h and w segments in the stream's table): a branch per pair on
+                            // the runtime segment widths serialises one load latency per pair
+                            const int pi0 = (cc & (p.head_dim - 1)) >> 1;
+                            const int dt2 = p.ra.dt2, dth = p.ra.dt2 + p.ra.dh2;
+                            const float2* t_row = s_t + f * dt2;
+                            const float2* h_row = p.ra.hw + rr * p.ra.dh2 - dt2;
+                            const float2* w_row = p.ra.hw + p.ra.gh * p.ra.dh2 + col * p.ra.dw2 - dth;
+                            float2 cs[16];
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) {
-                            const int pi = pi0 + i;
-                            const float2* src = pi < dt2 ? t_row + pi : (pi < dth ? h_row + pi : w_row + pi);
-                            cs[i] = *src;
+                            for (int i = 0; i < 16; ++i) {
+                                const int pi = pi0 + i;
+                                const float2* src = pi < dt2 ? t_row + pi : (pi < dth ? h_row + pi : w_row + pi);
+                                cs[i] = *src;
+                            }
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) w[i] = rope_pair(w[i], cs[i].x, cs[i].y);
                         }
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) w[i] = rope_pair(w[i], cs[i].x, cs[i].y);
+                        for (int i = 0; i < 4; ++i)
+                            st_shared_v4(rb + ((uint32_t(hh * 4 + i) ^ sw) << 4), w[4 * i], w[4 * i + 1],
+                                         w[4 * i + 2], w[4 * i + 3]);
                     }
-                    uint4* o = reinterpret_cast<uint4*>(dst + size_t(grow) * p.d + cc);
-#pragma unroll
-                    for (int i = 0; i < 4; ++i)
-                        o[i] = make_uint4(w[4 * i], w[4 * i + 1], w[4 * i + 2], w[4 * i + 3]);
-                    }
-                    __syncwarp();
+                    slab_release(&p.out_map[which], cbase + u * 64, tm * kBM);
                 }
             } else {
+                const int ucols = p.c_bf16 ? 64 : 32;      // output columns per unit
 #pragma unroll 1
-                for (int c = 0; c < BN / 32; ++c) {
-                    uint32_t r[32];
-                    tmem_ld32(tmem + lane_off + uint32_t(b * BN + c * 32), r);
-                    tmem_ld_wait();
-                    const int c0 = n0 + c * 32;
-                    if (live && c0 < p.N) {
-                    const size_t off = size_t(grow) * p.ldc + c0;
-                    if (c0 + 32 <= p.N) {
+                for (int u = 0; u < BN / ucols; ++u) {
+                    if (n0 + u * ucols >= p.N) break;       // the same for every thread
+                    slab_acquire();
+#pragma unroll 1
+                    for (int hh = 0; hh < ucols / 32; ++hh) {
+                        uint32_t r[32];
+                        tmem_ld32(tmem + lane_off + uint32_t(b * BN + u * ucols + hh * 32), r);
+                        tmem_ld_wait();
                         if (p.c_bf16) {
-                            uint4* o = reinterpret_cast<uint4*>(static_cast<uint16_t*>(p.c) + off);
 #pragma unroll
                             for (int i = 0; i < 4; ++i)
-                                o[i] = make_uint4(
-                                    pack_bf16x2(__uint_as_float(r[8 * i + 0]), __uint_as_float(r[8 * i + 1])),
-                                    pack_bf16x2(__uint_as_float(r[8 * i + 2]), __uint_as_float(r[8 * i + 3])),
-                                    pack_bf16x2(__uint_as_float(r[8 * i + 4]), __uint_as_float(r[8 * i + 5])),
-                                    pack_bf16x2(__uint_as_float(r[8 * i + 6]), __uint_as_float(r[8 * i + 7])));
+                                st_shared_v4(rb + ((uint32_t(hh * 4 + i) ^ sw) << 4),
+                                             pack_bf16x2(__uint_as_float(r[8 * i + 0]), __uint_as_float(r[8 * i + 1])),
+                                             pack_bf16x2(__uint_as_float(r[8 * i + 2]), __uint_as_float(r[8 * i + 3])),
+                                             pack_bf16x2(__uint_as_float(r[8 * i + 4]), __uint_as_float(r[8 * i + 5])),
+                                             pack_bf16x2(__uint_as_float(r[8 * i + 6]), __uint_as_float(r[8 * i + 7])));
                         } else {
-                            uint4* o = reinterpret_cast<uint4*>(static_cast<float*>(p.c) + off);
 #pragma unroll
                             for (int i = 0; i < 8; ++i)
-                                o[i] = make_uint4(r[4 * i], r[4 * i + 1], r[4 * i + 2], r[4 * i + 3]);
-                        }
-                    } else {
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) {
-                            if (c0 + i >= p.N) continue;
-                            const float v = __uint_as_float(r[i]);
-                            if (p.c_bf16) {
-                                static_cast<uint16_t*>(p.c)[off + i] =
-                                    uint16_t(pack_bf16x2(v, 0.0f) & 0xFFFFu);
-                            } else {
-                                static_cast<float*>(p.c)[off + i] = v;
-                            }
+                                st_shared_v4(rb + ((uint32_t(i) ^ sw) << 4), r[4 * i], r[4 * i + 1],
+                                             r[4 * i + 2], r[4 * i + 3]);
                         }
                     }
-                    }
-                    __syncwarp();
+                    slab_release(&p.out_map[0], n0 + u * ucols, tm * kBM);
                 }
             }
             tc_fence_before();
             if (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&bars.acc_empty[b]), 0));
             else mbar_arrive(smem_u32(&bars.acc_empty[b]));
         }
+        if (est) bulk_wait<0>();                       // C written before the CTA exits
     }
     __syncwarp();
     tc_fence_before();

@@ -109,6 +109,26 @@ frt_status make_part_map(CUtensorMap* map, float* base, int head_dim, long long 
     return FRT_OK;
 }
 
+// 2D store map over a row-major [rows, cols] fp32 or bf16 matrix with a leading dimension
+// of ld elements; box = 128 bytes of columns x 128 rows, 128-byte swizzle (the layout the
+// projection kernel stages its output units in); past the extent nothing is written.
+frt_status make_store_map_2d(CUtensorMap* map, void* base, long long cols, long long rows,
+                             long long ld, bool bf16) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return fail(FRT_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+    const int es = bf16 ? 2 : 4;
+    cuuint64_t dims[2] = {cuuint64_t(cols), cuuint64_t(rows)};
+    cuuint64_t strides[1] = {cuuint64_t(ld) * es};
+    cuuint32_t box[2] = {cuuint32_t(128 / es), 128};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = fn(map, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32,
+                    2, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                    CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(FRT_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", int(r));
+    return FRT_OK;
+}
+
 // 2D map over a row-major [rows, K] bf16 matrix; box = 64 columns x box_rows rows,
 // 128-byte swizzle; rows and columns past the extent read as zero.
 frt_status make_map_2d(CUtensorMap* map, const void* base, long long K, long long rows,
@@ -124,6 +144,37 @@ frt_status make_map_2d(CUtensorMap* map, const void* base, long long K, long lon
                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return fail(FRT_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", int(r));
     return FRT_OK;
+}
+
+// 3D view (64, rows, K / 64) of a row-major [rows, K] bf16 matrix (K a multiple of 64):
+// element (c, r, kb) is column 64 kb + c of row r, so one box (64, box_rows, 2) carries two
+// consecutive 64-column k-blocks of box_rows rows, laid out k-block after k-block.
+CUresult encode_kview(CUtensorMap* map, const void* base, long long K, long long rows,
+                      int box_rows) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return CUDA_ERROR_NOT_SUPPORTED;
+    cuuint64_t dims[3] = {64, cuuint64_t(rows), cuuint64_t(K / 64)};
+    cuuint64_t strides[2] = {cuuint64_t(K) * 2, 128};
+    cuuint32_t box[3] = {64, cuuint32_t(box_rows), 2};
+    cuuint32_t estr[3] = {1, 1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
+              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
+// Operand maps of C = A B^T (A [M, K], B [N, K] row-major bf16): k-block views when K is
+// a multiple of 64 and the driver takes them, else 2D maps (the kernel then issues one
+// copy per k-block).
+frt_status make_gemm_maps(GemmParams& g, const void* a, const void* b, long long K, long long M,
+                          long long N, int b_box_rows) {
+    if (K % 64 == 0 && encode_kview(&g.a_map, a, K, M, 128) == CUDA_SUCCESS &&
+        encode_kview(&g.b_map, b, K, N, b_box_rows) == CUDA_SUCCESS) {
+        g.kview3 = 1;
+        return FRT_OK;
+    }
+    g.kview3 = 0;
+    frt_status st = make_map_2d(&g.a_map, a, K, M, 128);
+    return st != FRT_OK ? st : make_map_2d(&g.b_map, b, K, N, b_box_rows);
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
@@ -636,8 +687,7 @@ frt_status frt_block_step(frt_stream_t* s, const void* x, const void* w_qkv, con
     GemmParams g;
     std::memset(&g, 0, sizeof(g));
     const int bn = gemm_block_n_for(s->n_q, 3 * d, kEpiQkv, d);
-    if ((st = make_map_2d(&g.a_map, x, d, s->n_q, 128)) != FRT_OK) return st;
-    if ((st = make_map_2d(&g.b_map, w_qkv, d, 3LL * d, bn / gemm_cluster_m(s->n_q))) != FRT_OK)
+    if ((st = make_gemm_maps(g, x, w_qkv, d, s->n_q, 3LL * d, bn / gemm_cluster_m(s->n_q))) != FRT_OK)
         return st;
     g.M = s->n_q;
     g.N = 3 * d;
@@ -648,6 +698,10 @@ frt_status frt_block_step(frt_stream_t* s, const void* x, const void* w_qkv, con
     g.q_out = static_cast<uint16_t*>(q_buf);
     g.k_out = static_cast<uint16_t*>(s->cache_k) + off;
     g.v_out = static_cast<uint16_t*>(s->cache_v) + off;
+    if ((st = make_store_map_2d(&g.out_map[0], g.q_out, d, s->n_q, d, true)) != FRT_OK ||
+        (st = make_store_map_2d(&g.out_map[1], g.k_out, d, s->n_q, d, true)) != FRT_OK ||
+        (st = make_store_map_2d(&g.out_map[2], g.v_out, d, s->n_q, d, true)) != FRT_OK)
+        return st;
     g.rope = 1;
     fill_rope(s, s->counter, g.ra);
     g.wait_limit_ns = s->wait_limit_ns;
@@ -672,8 +726,8 @@ frt_status frt_block_step(frt_stream_t* s, const void* x, const void* w_qkv, con
     GemmParams h;
     std::memset(&h, 0, sizeof(h));
     const int bn2 = gemm_block_n_for(s->n_q, d, kEpiPlain, 0);
-    if ((st = make_map_2d(&h.a_map, o_buf, d, s->n_q, 128)) != FRT_OK) return st;
-    if ((st = make_map_2d(&h.b_map, w_o, d, d, bn2 / gemm_cluster_m(s->n_q))) != FRT_OK) return st;
+    if ((st = make_gemm_maps(h, o_buf, w_o, d, s->n_q, d, bn2 / gemm_cluster_m(s->n_q))) != FRT_OK)
+        return st;
     h.M = s->n_q;
     h.N = d;
     h.K = d;
@@ -681,6 +735,7 @@ frt_status frt_block_step(frt_stream_t* s, const void* x, const void* w_qkv, con
     h.c = y;
     h.ldc = d;
     h.c_bf16 = s->cfg.out_dtype == FRT_OUT_BF16;
+    if ((st = make_store_map_2d(&h.out_map[0], y, d, s->n_q, d, h.c_bf16 != 0)) != FRT_OK) return st;
     h.wait_limit_ns = s->wait_limit_ns;
     h.status = s->status_dev;
     if (s->proj_start) e = cudaEventRecord(s->proj_start, s->cs);
@@ -705,8 +760,7 @@ frt_status frt_gemm_bf16(const void* a, const void* b, void* c, int M, int N, in
     GemmParams g;
     std::memset(&g, 0, sizeof(g));
     frt_status st;
-    if ((st = make_map_2d(&g.a_map, a, K, M, 128)) != FRT_OK) return st;
-    if ((st = make_map_2d(&g.b_map, b, K, N, gemm_block_n_for(M, N, kEpiPlain, 0) / gemm_cluster_m(M))) !=
+    if ((st = make_gemm_maps(g, a, b, K, M, N, gemm_block_n_for(M, N, kEpiPlain, 0) / gemm_cluster_m(M))) !=
         FRT_OK)
         return st;
     g.M = M;
@@ -716,6 +770,7 @@ frt_status frt_gemm_bf16(const void* a, const void* b, void* c, int M, int N, in
     g.c = c;
     g.ldc = ldc;
     g.c_bf16 = c_dtype == FRT_OUT_BF16;
+    if ((st = make_store_map_2d(&g.out_map[0], c, N, M, ldc, g.c_bf16 != 0)) != FRT_OK) return st;
     g.wait_limit_ns = kDefaultWaitLimitNs;
     g.status = static_cast<DeviceStatus*>(status);
     cudaError_t e = launch_gemm(g, static_cast<cudaStream_t>(cuda_stream));

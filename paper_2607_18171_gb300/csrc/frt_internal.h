@@ -138,8 +138,12 @@ constexpr int kEpiPlain = 0;   // C row-major, fp32 or bf16
 constexpr int kEpiQkv = 1;     // DiT-block QKV projection: q -> q_out, k/v -> cache slot
 
 struct GemmParams {
-    CUtensorMap a_map;      // 2D (K, M) bf16, box (64, 128), 128-byte swizzle
-    CUtensorMap b_map;      // 2D (K, N) bf16, box (64, BN), 128-byte swizzle
+    CUtensorMap a_map;      // 3D (64, M, K / 64) bf16, box (64, 128, 2) when kview3, else
+                            // 2D (K, M), box (64, 128); 128-byte swizzle
+    CUtensorMap b_map;      // the same over B [N, K], box rows BN / CTAs per tile
+    CUtensorMap out_map[3]; // TMA store maps, 128-byte swizzle, box (128 bytes of columns,
+                            // 128 rows): plain [0] over C (N, M); QKV [0..2] over q, k, v (d, M)
+    int kview3;             // both maps are 3D k-block views (K a multiple of 64)
     int M, N, K;
     int tiles_m, tiles_n;   // filled in by launch_gemm
     int epi;

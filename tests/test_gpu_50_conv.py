@@ -198,3 +198,12 @@ def test_conv_rejects_bad_arguments(frt):
         with pytest.raises(frt.FrtError):
             st.set_tile(bn, pr)
     st.close()
+    # a bf16 output is staged in 64-channel units: a 96-wide tile cannot write it
+    cw = SMALL["conv_kt1"]
+    st = frt.ConvStream(cw.cin, cw.cout, cw.kt, cw.kh, cw.kw, cw.grid_h, cw.grid_w, cw.frames,
+                        out_dtype=torch.bfloat16)
+    w, b = (t.cuda() for t in synth.conv_weights(cw))
+    st.set_tile(96, 1)
+    with pytest.raises(frt.FrtError):
+        st.step(synth.conv_chunk(cw, 0, 0).cuda(), w, b, st.new_out())
+    st.close()
