@@ -383,10 +383,12 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
             tc_fence_after();
 #pragma unroll 1
             for (int u = 0; u < BN / ucols; ++u) {
-                if (est) bulk_wait_read<0>();            // the previous store has read the slab
-                named_bar_sync(1, 128);
-#pragma unroll 1
-                for (int h = 0; h < ucols / 32; ++h) {
+                // the unit's 32 words per thread are computed before the slab is claimed,
+                // so the previous store's read of the slab overlaps this work
+                uint32_t o[32];
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    if (h == 1 && !p.y_bf16) break;
                     const int c = u * ucols + h * 32;    // first column of this TMEM load
                     uint32_t r[32];
                     tmem_ld32(tmem + lane_off + uint32_t(b * BN + c), r);
@@ -403,18 +405,18 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
                     }
                     if (p.y_bf16) {
 #pragma unroll
-                        for (int i = 0; i < 4; ++i)
-                            st_shared_v4(rb + ((uint32_t(h * 4 + i) ^ sw) << 4),
-                                         pack_bf16x2(v[8 * i], v[8 * i + 1]), pack_bf16x2(v[8 * i + 2], v[8 * i + 3]),
-                                         pack_bf16x2(v[8 * i + 4], v[8 * i + 5]), pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
+                        for (int i = 0; i < 16; ++i) o[16 * h + i] = pack_bf16x2(v[2 * i], v[2 * i + 1]);
                     } else {
 #pragma unroll
-                        for (int i = 0; i < 8; ++i)
-                            st_shared_v4(rb + ((uint32_t(i) ^ sw) << 4), __float_as_uint(v[4 * i]),
-                                         __float_as_uint(v[4 * i + 1]), __float_as_uint(v[4 * i + 2]),
-                                         __float_as_uint(v[4 * i + 3]));
+                        for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(v[i]);
                     }
                 }
+                if (est) bulk_wait_read<0>();            // the previous store has read the slab
+                named_bar_sync(1, 128);
+#pragma unroll
+                for (int i = 0; i < 8; ++i)
+                    st_shared_v4(rb + ((uint32_t(i) ^ sw) << 4), o[4 * i], o[4 * i + 1], o[4 * i + 2],
+                                 o[4 * i + 3]);
                 fence_proxy_async_smem();
                 named_bar_sync(1, 128);
                 if (est && f < p.F) {

@@ -313,15 +313,17 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
                 }
 #pragma unroll 1
                 for (int u = 0; u < BN / 64; ++u) {      // 64 bf16 columns per unit
-                    slab_acquire();
-#pragma unroll 1
+                    // the unit's values are computed before the slab is claimed, so the
+                    // previous store's read of the slab overlaps this work
+                    uint32_t wu[2][16];
+#pragma unroll
                     for (int hh = 0; hh < 2; ++hh) {
                         const int c = 2 * u + hh;
                         uint32_t r[32];
                         tmem_ld32(tmem + lane_off + uint32_t(b * BN + c * 32), r);
                         tmem_ld_wait();
                         const int cc = cbase + c * 32;
-                        uint32_t w[16];
+                        uint32_t (&w)[16] = wu[hh];
 #pragma unroll
                         for (int i = 0; i < 16; ++i)
                             w[i] = pack_bf16x2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
@@ -345,11 +347,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
 #pragma unroll
                             for (int i = 0; i < 16; ++i) w[i] = rope_pair(w[i], cs[i].x, cs[i].y);
                         }
+                    }
+                    slab_acquire();
+#pragma unroll
+                    for (int hh = 0; hh < 2; ++hh)
 #pragma unroll
                         for (int i = 0; i < 4; ++i)
-                            st_shared_v4(rb + ((uint32_t(hh * 4 + i) ^ sw) << 4), w[4 * i], w[4 * i + 1],
-                                         w[4 * i + 2], w[4 * i + 3]);
-                    }
+                            st_shared_v4(rb + ((uint32_t(hh * 4 + i) ^ sw) << 4), wu[hh][4 * i],
+                                         wu[hh][4 * i + 1], wu[hh][4 * i + 2], wu[hh][4 * i + 3]);
                     slab_release(&p.out_map[which], cbase + u * 64, tm * kBM);
                 }
             } else {
@@ -357,27 +362,27 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
 #pragma unroll 1
                 for (int u = 0; u < BN / ucols; ++u) {
                     if (n0 + u * ucols >= p.N) break;       // the same for every thread
-                    slab_acquire();
-#pragma unroll 1
-                    for (int hh = 0; hh < ucols / 32; ++hh) {
-                        uint32_t r[32];
-                        tmem_ld32(tmem + lane_off + uint32_t(b * BN + u * ucols + hh * 32), r);
-                        tmem_ld_wait();
-                        if (p.c_bf16) {
+                    // 32 words per thread per unit, loaded before the slab is claimed
+                    uint32_t v[32];
+                    if (p.c_bf16) {
 #pragma unroll
-                            for (int i = 0; i < 4; ++i)
-                                st_shared_v4(rb + ((uint32_t(hh * 4 + i) ^ sw) << 4),
-                                             pack_bf16x2(__uint_as_float(r[8 * i + 0]), __uint_as_float(r[8 * i + 1])),
-                                             pack_bf16x2(__uint_as_float(r[8 * i + 2]), __uint_as_float(r[8 * i + 3])),
-                                             pack_bf16x2(__uint_as_float(r[8 * i + 4]), __uint_as_float(r[8 * i + 5])),
-                                             pack_bf16x2(__uint_as_float(r[8 * i + 6]), __uint_as_float(r[8 * i + 7])));
-                        } else {
+                        for (int hh = 0; hh < 2; ++hh) {
+                            uint32_t r[32];
+                            tmem_ld32(tmem + lane_off + uint32_t(b * BN + u * ucols + hh * 32), r);
+                            tmem_ld_wait();
 #pragma unroll
-                            for (int i = 0; i < 8; ++i)
-                                st_shared_v4(rb + ((uint32_t(i) ^ sw) << 4), r[4 * i], r[4 * i + 1],
-                                             r[4 * i + 2], r[4 * i + 3]);
+                            for (int i = 0; i < 16; ++i)
+                                v[16 * hh + i] = pack_bf16x2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
                         }
+                    } else {
+                        tmem_ld32(tmem + lane_off + uint32_t(b * BN + u * ucols), v);
+                        tmem_ld_wait();
                     }
+                    slab_acquire();
+#pragma unroll
+                    for (int i = 0; i < 8; ++i)
+                        st_shared_v4(rb + ((uint32_t(i) ^ sw) << 4), v[4 * i], v[4 * i + 1], v[4 * i + 2],
+                                     v[4 * i + 3]);
                     slab_release(&p.out_map[0], n0 + u * ucols, tm * kBM);
                 }
             }
