@@ -488,6 +488,14 @@ BLOCK_METRIC = ("DiT-block attention-slice TFLOP/s (QKV projection + RoPE + KV a
                 "chunk attention + output projection) per frame-chunk at 1 GB300")
 
 
+def gemm_label(M, N, qkv, d, what):
+    """Name of the projection kernel instance the library picks for C [M, N]."""
+    from paper_2607_18171_gb300 import frt
+
+    bn, ctas = frt.gemm_plan(M, N, qkv, d)
+    return f"gemm_kernel<{bn}, {'pair' if ctas == 2 else 'single'}> ({what})"
+
+
 def run_gpu_block(args, wl, world, rank, local, dev, peak_tf, peak_kind):
     """One DiT block's attention slice per step (frt_block_step: QKV projection with
     RoPE and the append in its epilogue, chunk attention, output projection) at steady
@@ -569,10 +577,11 @@ def run_gpu_block(args, wl, world, rank, local, dev, peak_tf, peak_kind):
                      "kernel": "attn_kernel<128,1,false>", "peak_kind": peak_kind,
                      "launch_ms": round(attn_ms, 4)},
         "projections": {
-            "qkv": {"kernel": "gemm_kernel<256> (QKV epilogue)", "launch_ms": round(qkv_ms, 4),
+            "qkv": {"kernel": gemm_label(wl.n_q, 3 * d, True, d, "QKV epilogue"),
+                    "launch_ms": round(qkv_ms, 4),
                     "achieved": round(tf(qkv_flops, qkv_ms), 2),
                     "frac": round(tf(qkv_flops, qkv_ms) / peak_tf, 4)},
-            "out": {"kernel": "gemm_kernel<256> (plain epilogue, fp32 out)",
+            "out": {"kernel": gemm_label(wl.n_q, d, False, 0, "plain epilogue, fp32 out"),
                     "launch_ms": round(out_ms, 4), "achieved": round(tf(out_flops, out_ms), 2),
                     "frac": round(tf(out_flops, out_ms) / peak_tf, 4)},
             "unit": "TFLOP/s", "peak": peak_tf},

@@ -162,6 +162,13 @@ frt_status frt_block_step(frt_stream_t* s, const void* x, const void* w_qkv,
 frt_status frt_gemm_bf16(const void* a, const void* b, void* c, int M, int N,
                          int K, int ldc, int c_dtype, void* status,
                          void* cuda_stream);
+/* Tile plan of the projection kernel for C [M, N] (for reports; no counterpart in the
+ * paper): *bn = output columns per tile (128 or 256), *ctas = CTAs per tile (2: a CTA
+ * pair on 256 rows, 1: one CTA on 128 rows). qkv = 1 asks for the QKV epilogue of
+ * frt_block_step with d = heads * head_dim (N = 3 d). FRT_ERR_INVALID_ARG on NULL
+ * outputs or non-positive sizes. Host-only: it launches nothing and reads only the
+ * current device's SM count (148 assumed when no device is visible). */
+frt_status frt_gemm_plan(int M, int N, int qkv, int d, int* bn, int* ctas);
 
 /* ---- Streaming causal 3D convolution (the VAE-decoder stage) --------------------
  * The paper's video pipelines end in a streaming VAE decoder (Appendix A.3, the

@@ -745,6 +745,14 @@ frt_status frt_block_step(frt_stream_t* s, const void* x, const void* w_qkv, con
     return FRT_OK;
 }
 
+frt_status frt_gemm_plan(int M, int N, int qkv, int d, int* bn, int* ctas) {
+    if (!bn || !ctas || M < 1 || N < 1 || (qkv && d < 1))
+        return fail(FRT_ERR_INVALID_ARG, "need bn, ctas non-NULL and positive sizes");
+    *bn = gemm_block_n_for(M, N, qkv ? kEpiQkv : kEpiPlain, qkv ? d : 0);
+    *ctas = gemm_cluster_m(M);
+    return FRT_OK;
+}
+
 frt_status frt_gemm_bf16(const void* a, const void* b, void* c, int M, int N, int K, int ldc,
                          int c_dtype, void* status, void* cuda_stream) {
     if (!a || !b || !c || !aligned16(a) || !aligned16(b) || !aligned16(c) ||

@@ -76,6 +76,7 @@ def lib() -> ctypes.CDLL:
         "frt_conv_reset": (I, [P]),
         "frt_conv_destroy": (None, [P]),
         "frt_gemm_bf16": (I, [P, P, P, I, I, I, I, I, P, P]),
+        "frt_gemm_plan": (I, [I, I, I, I, ctypes.POINTER(I), ctypes.POINTER(I)]),
         "frt_stream_set_block_events": (I, [P, P, P, P, P]),
         "frt_window_index": (I, [LL, I, ctypes.POINTER(I), ctypes.POINTER(LL),
                                  ctypes.POINTER(I)]),
@@ -419,6 +420,13 @@ class Steps:
             self.close()
         except Exception:
             pass
+
+
+def gemm_plan(M: int, N: int, qkv: bool = False, d: int = 0) -> tuple[int, int]:
+    """(output columns per tile, CTAs per tile) the projection kernel uses for C [M, N]."""
+    bn, ctas = ctypes.c_int(), ctypes.c_int()
+    _check(lib().frt_gemm_plan(M, N, 1 if qkv else 0, d, ctypes.byref(bn), ctypes.byref(ctas)))
+    return bn.value, ctas.value
 
 
 def gemm_bf16(a: torch.Tensor, b: torch.Tensor, c: torch.Tensor,

@@ -131,3 +131,17 @@ def test_step_group_argument_checks(frt):
     assert L.frt_steps_tick(g, 0b1000, arr, arr, arr, arr) == 1
     L.frt_steps_destroy(g)
     L.frt_steps_destroy(None)
+
+
+def test_gemm_plan_is_host_only_and_checks_arguments(frt):
+    # one 128-row tile: a single CTA; two or more: a CTA pair on 256 rows
+    assert frt.gemm_plan(128, 1536)[1] == 1
+    assert frt.gemm_plan(4680, 1536)[1] == 2
+    for M, N, qkv, d in ((4680, 1536, False, 0), (4680, 4608, True, 1536), (300, 200, False, 0)):
+        bn, ctas = frt.gemm_plan(M, N, qkv, d)
+        assert bn in (128, 256) and ctas in (1, 2)
+    # the QKV epilogue needs 128-wide tiles unless d is a multiple of 256
+    assert frt.gemm_plan(4680, 3 * 640, True, 640)[0] == 128
+    for args in ((0, 16, False, 0), (16, 0, False, 0), (16, 48, True, 0)):
+        with pytest.raises(frt.FrtError):
+            frt.gemm_plan(*args)
