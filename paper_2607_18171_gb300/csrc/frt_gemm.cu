@@ -442,8 +442,8 @@ int gemm_cluster_m(int M) { return M > kBM ? 2 : 1; }
 int gemm_block_n(int N, int epi, int d) {
     // 128-column tiles when the QKV epilogue needs them (d not a multiple of 256) or N
     // is small; otherwise 256 unless 128 balances the rounds of tiles over the SMs
-    // clearly better (tile cost ~ BN, plus a quarter at 128 for the higher operand
-    // traffic per FLOP)
+    // clearly better (tile cost ~ BN, times 1.5 at 128: measured, an N = 128 MMA of a CTA
+    // pair issues in ~82 cycles for 64 of work and its stage waits are exposed)
     if (epi == kEpiQkv && d % 256 != 0) return 128;
     if (N <= 128) return 128;
     (void)d;
@@ -457,7 +457,7 @@ int gemm_block_n_for(int M, int N, int epi, int d) {
     const long long ctm = ((M + kBM - 1) / kBM + gemm_cluster_m(M) - 1) / gemm_cluster_m(M);
     const long long r256 = (ctm * ((N + 255) / 256) + units - 1) / units;
     const long long r128 = (ctm * ((N + 127) / 128) + units - 1) / units;
-    return (r128 * 128 * 5 < r256 * 256 * 4) ? 128 : 256;
+    return (r128 * 128 * 3 < r256 * 256 * 2) ? 128 : 256;
 }
 
 cudaError_t launch_gemm(GemmParams p, cudaStream_t st) {
