@@ -2,7 +2,7 @@
 // fp32 accumulation in TMEM, for the linear projections around the chunk attention of a
 // DiT block (QKV projection in front of it, output projection after it).
 //
-// Persistent kernel, one CTA per SM, 192 threads:
+// Persistent kernel, one CTA per SM, 320 threads:
 //   warp 0      TMA producer: two k-blocks of A (128 x 64 each) and of B (BN x 64 each)
 //               per ring stage, 128-byte swizzle, through a shared-memory ring (with K a
 //               multiple of 64, one box per operand loads both k-blocks through a 3D view
@@ -11,9 +11,9 @@
 //               per instruction, eight per stage: one barrier wait per eight MMAs, since a
 //               shared-memory access by the issuing thread behind queued MMAs stalls it
 //               ~140 cycles);
-//   warps 2-5   epilogue: one thread per accumulator row (TMEM lane), 32 columns per
-//               tcgen05.ld; each 128-byte column unit of the tile (32 fp32 or 64 bf16
-//               columns) is staged in a 128-byte-swizzled shared-memory slab and written
+//   warps 2-9   epilogue: two warps per TMEM lane quarter, each thread one accumulator
+//               row (TMEM lane) and one half of every column unit: each 128-byte
+//               column unit of the tile (32 fp32 or 64 bf16 columns) is staged in a 128-byte-swizzled shared-memory slab and written
 //               by one TMA tensor store (rows past M and columns past N are clipped by
 //               the store); per-thread row stores would touch 32 rows per warp
 //               instruction.
@@ -46,7 +46,8 @@ namespace frt {
 
 namespace {
 
-constexpr int kThreads = 192;
+constexpr int kThreads = 320;
+constexpr int kEpiThreads = 256;   // warps 2-9
 constexpr int kBM = 128;
 constexpr int kBK = 64;          // one 128-byte swizzle atom of bf16
 constexpr int kMaxStages = 6;
@@ -122,7 +123,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_u32(&bars.acc_full[b]), 1);
-            mbar_init(smem_u32(&bars.acc_empty[b]), 128 * CM);
+            mbar_init(smem_u32(&bars.acc_empty[b]), kEpiThreads * CM);
         }
         mbar_init(smem_u32(&bars.drain), 1);
         bars.abort_flag = 0;
@@ -266,6 +267,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
     } else {
         // ====================================== epilogue =====================================
         const int sub = warp & 3;                      // TMEM lane quarter of this warp
+        const int half = (warp - 2) >> 2;              // which half of each column unit
         const int row = sub * 32 + lane;
         const uint32_t lane_off = uint32_t(sub * 32) << 16;
         const uint32_t stg = sbase + uint32_t(kStages * C::STAGE);   // 1024-aligned slab
@@ -275,11 +277,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
         // slab free (the previous store has read it), then every thread refills it
         auto slab_acquire = [&]() {
             if (est) bulk_wait_read<0>();
-            named_bar_sync(1, 128);
+            named_bar_sync(1, kEpiThreads);
         };
         auto slab_release = [&](const CUtensorMap* map, int c0, int r0) {
             fence_proxy_async_smem();
-            named_bar_sync(1, 128);
+            named_bar_sync(1, kEpiThreads);
             if (est) {
                 tma_store_2d(map, stg, c0, r0);
                 bulk_commit();
@@ -291,8 +293,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
             const int tm = (t % ctm) * CM + rank;
             const int tn = t / ctm;
             const bool got = mbar_wait(smem_u32(&bars.acc_full[b]), (tl >> 1) & 1, lim, abort);
-            // all four warps go on or stop together: the staging below synchronises them
-            if (!named_bar_and(1, 128, got)) {
+            // all epilogue warps go on or stop together: the staging below synchronises them
+            if (!named_bar_and(1, kEpiThreads, got)) {
                 if (!got) report(p.status, abort, 2, tl);
                 break;
             }
@@ -315,10 +317,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
                 for (int u = 0; u < BN / 64; ++u) {      // 64 bf16 columns per unit
                     // the unit's values are computed before the slab is claimed, so the
                     // previous store's read of the slab overlaps this work
-                    uint32_t wu[2][16];
-#pragma unroll
-                    for (int hh = 0; hh < 2; ++hh) {
-                        const int c = 2 * u + hh;
+                    uint32_t wu[1][16];
+                    {
+                        const int hh = 0;
+                        const int c = 2 * u + half;               // this half's 32 columns
                         uint32_t r[32];
                         tmem_ld32(tmem + lane_off + uint32_t(b * BN + c * 32), r);
                         tmem_ld_wait();
@@ -350,11 +352,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
                     }
                     slab_acquire();
 #pragma unroll
-                    for (int hh = 0; hh < 2; ++hh)
-#pragma unroll
-                        for (int i = 0; i < 4; ++i)
-                            st_shared_v4(rb + ((uint32_t(hh * 4 + i) ^ sw) << 4), wu[hh][4 * i],
-                                         wu[hh][4 * i + 1], wu[hh][4 * i + 2], wu[hh][4 * i + 3]);
+                    for (int i = 0; i < 4; ++i)
+                        st_shared_v4(rb + ((uint32_t(half * 4 + i) ^ sw) << 4), wu[0][4 * i],
+                                     wu[0][4 * i + 1], wu[0][4 * i + 2], wu[0][4 * i + 3]);
                     slab_release(&p.out_map[which], cbase + u * 64, tm * kBM);
                 }
             } else {
@@ -362,27 +362,25 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
 #pragma unroll 1
                 for (int u = 0; u < BN / ucols; ++u) {
                     if (n0 + u * ucols >= p.N) break;       // the same for every thread
-                    // 32 words per thread per unit, loaded before the slab is claimed
-                    uint32_t v[32];
+                    // this half's 64 bytes of the row (16 words), loaded before the slab
+                    // is claimed
+                    uint32_t v[16];
                     if (p.c_bf16) {
+                        uint32_t r[32];
+                        tmem_ld32(tmem + lane_off + uint32_t(b * BN + u * ucols + half * 32), r);
+                        tmem_ld_wait();
 #pragma unroll
-                        for (int hh = 0; hh < 2; ++hh) {
-                            uint32_t r[32];
-                            tmem_ld32(tmem + lane_off + uint32_t(b * BN + u * ucols + hh * 32), r);
-                            tmem_ld_wait();
-#pragma unroll
-                            for (int i = 0; i < 16; ++i)
-                                v[16 * hh + i] = pack_bf16x2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
-                        }
+                        for (int i = 0; i < 16; ++i)
+                            v[i] = pack_bf16x2(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
                     } else {
-                        tmem_ld32(tmem + lane_off + uint32_t(b * BN + u * ucols), v);
+                        tmem_ld16(tmem + lane_off + uint32_t(b * BN + u * ucols + half * 16), v);
                         tmem_ld_wait();
                     }
                     slab_acquire();
 #pragma unroll
-                    for (int i = 0; i < 8; ++i)
-                        st_shared_v4(rb + ((uint32_t(i) ^ sw) << 4), v[4 * i], v[4 * i + 1], v[4 * i + 2],
-                                     v[4 * i + 3]);
+                    for (int i = 0; i < 4; ++i)
+                        st_shared_v4(rb + ((uint32_t(half * 4 + i) ^ sw) << 4), v[4 * i], v[4 * i + 1],
+                                     v[4 * i + 2], v[4 * i + 3]);
                     slab_release(&p.out_map[0], n0 + u * ucols, tm * kBM);
                 }
             }
