@@ -33,6 +33,12 @@ int frt_selftest_umma_tile(const void* a, const void* b, float* c, int b_mn_majo
 int frt_selftest_umma_pair(const void* a, const void* b, float* c, unsigned* taddrs,
                            int* dev_status, void* cuda_stream);
 
+/* Force the output-column tile width of every later projection launch (frt_gemm_bf16,
+ * frt_block_step, frt_gemm_plan) to bn in {128, 192, 256}; 0 restores the automatic
+ * choice. Process-wide and not thread-safe: for tests that cover every width. Returns
+ * 0, or -1 for another value. */
+int frt_selftest_gemm_force_bn(int bn);
+
 /* Launch a kernel whose one waiting thread waits on an mbarrier that nothing arrives
  * on, bounded by limit_ns (<= 100 ms); it must record FRT_ERR_TIMEOUT in s's status
  * block, which frt_stream_sync then returns. s must be configured. */

@@ -65,7 +65,7 @@ struct GCfg {
                                       ? (225 * 1024 - 1024 - SLAB) / STAGE : kMaxStages;
     static constexpr int SMEM = STAGES * STAGE + SLAB + 1024;   // + alignment slack
     static constexpr uint32_t IDESC = idesc_bf16_f32(kBM * CM, BN, false);
-    static constexpr uint32_t TMEM_COLS = 2 * BN;
+    static constexpr uint32_t TMEM_COLS = 2 * BN <= 256 ? 256 : 512;   // a power of two
 };
 
 struct GBars {
@@ -437,25 +437,31 @@ cudaError_t launch(const GemmParams& p, cudaStream_t st) {
 // CTAs per tile: a pair (cta_group::2) whenever there are at least two M tiles.
 int gemm_cluster_m(int M) { return M > kBM ? 2 : 1; }
 
-int gemm_block_n(int N, int epi, int d) {
-    // 128-column tiles when the QKV epilogue needs them (d not a multiple of 256) or N
-    // is small; otherwise 256 unless 128 balances the rounds of tiles over the SMs
-    // clearly better (tile cost ~ BN, times 1.5 at 128: measured, an N = 128 MMA of a CTA
-    // pair issues in ~82 cycles for 64 of work and its stage waits are exposed)
-    if (epi == kEpiQkv && d % 256 != 0) return 128;
-    if (N <= 128) return 128;
-    (void)d;
-    return 256;
-}
+// Output columns per tile: the width in {128, 192, 256} with the least rounds of tiles
+// over the SMs (or SM pairs) x width, a 128-wide tile weighted 1.5x (measured: an N = 128
+// MMA of a CTA pair issues in ~82 cycles for 64 of work and its stage waits are exposed).
+// The QKV epilogue needs a width dividing d (a tile never straddles q, k and v); widths
+// past N are not considered unless nothing else fits.
+int g_force_bn = 0;   // test override (frt_selftest_gemm_force_bn)
 
 int gemm_block_n_for(int M, int N, int epi, int d) {
-    const int bn = gemm_block_n(N, epi, d);
-    if (bn == 128 || (epi == kEpiQkv && d % 128 != 0)) return bn;
-    const int units = num_sms() / gemm_cluster_m(M);
-    const long long ctm = ((M + kBM - 1) / kBM + gemm_cluster_m(M) - 1) / gemm_cluster_m(M);
-    const long long r256 = (ctm * ((N + 255) / 256) + units - 1) / units;
-    const long long r128 = (ctm * ((N + 127) / 128) + units - 1) / units;
-    return (r128 * 128 * 3 < r256 * 256 * 2) ? 128 : 256;
+    if (g_force_bn != 0) return g_force_bn;
+    const int cm = gemm_cluster_m(M);
+    const long long units = num_sms() / cm;
+    const long long ctm = ((M + kBM - 1) / kBM + cm - 1) / cm;
+    int best = 128;
+    double best_t = 1e30;
+    for (int bn : {256, 192, 128}) {
+        if (epi == kEpiQkv && d % bn != 0) continue;
+        if (bn > 128 && bn > N) continue;
+        const long long tiles = ctm * ((N + bn - 1) / bn);
+        const double t = double((tiles + units - 1) / units) * bn * (bn == 128 ? 1.5 : 1.0);
+        if (t < best_t - 1e-9) {
+            best_t = t;
+            best = bn;
+        }
+    }
+    return best;
 }
 
 cudaError_t launch_gemm(GemmParams p, cudaStream_t st) {
@@ -464,8 +470,16 @@ cudaError_t launch_gemm(GemmParams p, cudaStream_t st) {
     p.tiles_m = (p.M + kBM - 1) / kBM;
     p.tiles_n = (p.N + bn - 1) / bn;
     if (gemm_cluster_m(p.M) == 2)
-        return bn == 256 ? launch<256, true>(p, st) : launch<128, true>(p, st);
-    return bn == 256 ? launch<256, false>(p, st) : launch<128, false>(p, st);
+        return bn == 256 ? launch<256, true>(p, st)
+                         : (bn == 192 ? launch<192, true>(p, st) : launch<128, true>(p, st));
+    return bn == 256 ? launch<256, false>(p, st)
+                     : (bn == 192 ? launch<192, false>(p, st) : launch<128, false>(p, st));
 }
 
 }  // namespace frt
+
+extern "C" int frt_selftest_gemm_force_bn(int bn) {
+    if (bn != 0 && bn != 128 && bn != 192 && bn != 256) return -1;
+    frt::g_force_bn = bn;
+    return 0;
+}

@@ -86,6 +86,7 @@ def lib() -> ctypes.CDLL:
         "frt_selftest_umma_tile": (I, [P, P, P, I, I, I, I, P, P]),
         "frt_selftest_wait_timeout": (I, [P, LL, P]),
         "frt_selftest_umma_pair": (I, [P, P, P, P, P, P]),
+        "frt_selftest_gemm_force_bn": (I, [I]),
         "frt_steps_create": (P, [I, I, I, I, I, I]),
         "frt_steps_configure": (I, [P, ctypes.POINTER(Config)]),
         "frt_steps_stream": (P, [P, I]),
@@ -420,6 +421,12 @@ class Steps:
             self.close()
         except Exception:
             pass
+
+
+def selftest_gemm_force_bn(bn: int) -> None:
+    """Force the projection kernel's tile width (128, 192 or 256; 0 = automatic)."""
+    if lib().frt_selftest_gemm_force_bn(bn) != 0:
+        raise ValueError("bn must be 0, 128, 192 or 256")
 
 
 def gemm_plan(M: int, N: int, qkv: bool = False, d: int = 0) -> tuple[int, int]:

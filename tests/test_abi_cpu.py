@@ -139,9 +139,10 @@ def test_gemm_plan_is_host_only_and_checks_arguments(frt):
     assert frt.gemm_plan(4680, 1536)[1] == 2
     for M, N, qkv, d in ((4680, 1536, False, 0), (4680, 4608, True, 1536), (300, 200, False, 0)):
         bn, ctas = frt.gemm_plan(M, N, qkv, d)
-        assert bn in (128, 256) and ctas in (1, 2)
-    # the QKV epilogue needs 128-wide tiles unless d is a multiple of 256
+        assert bn in (128, 192, 256) and ctas in (1, 2)
+    # a QKV tile never straddles q, k and v: its width divides d
     assert frt.gemm_plan(4680, 3 * 640, True, 640)[0] == 128
+    assert 1536 % frt.gemm_plan(4680, 3 * 1536, True, 1536)[0] == 0
     for args in ((0, 16, False, 0), (16, 0, False, 0), (16, 48, True, 0)):
         with pytest.raises(frt.FrtError):
             frt.gemm_plan(*args)

@@ -59,6 +59,29 @@ def test_gemm_matches_fp64(frt, M, N, K, out):
     assert np.all(got[:, N:] == 7.0)
 
 
+@pytest.mark.parametrize("bn", [128, 192, 256])
+@pytest.mark.parametrize("M,N,K", [(300, 200, 136), (1000, 384, 512), (96, 4608, 1536),
+                                   (4680, 1536, 1536)])
+def test_gemm_every_tile_width_matches_fp64(frt, M, N, K, bn):
+    """Every output-column tile width, single CTAs (M <= 128) and CTA pairs, 2D and 3D
+    operand views (K % 64), ragged M, N and K against the same bound."""
+    g = torch.Generator().manual_seed(M * 5 + N + K + bn)
+    a = torch.randn(M, K, generator=g).to(torch.bfloat16)
+    b = (torch.randn(N, K, generator=g) * K ** -0.5).to(torch.bfloat16)
+    c = torch.full((M, N), 7.0, dtype=torch.float32, device="cuda")
+    frt.selftest_gemm_force_bn(bn)
+    try:
+        assert frt.gemm_plan(M, N)[0] == bn
+        frt.gemm_bf16(a.cuda(), b.cuda(), c)
+        torch.cuda.synchronize()
+    finally:
+        frt.selftest_gemm_force_bn(0)
+    af, bf = _f64(a), _f64(b)
+    err = np.abs(_f64(c) - linear(af, bf))
+    bound = _gemm_bound(af, bf)
+    assert np.all(err <= bound + 1e-30), f"bn {bn}: max excess {float(np.max(err - bound)):.3e}"
+
+
 def test_gemm_is_deterministic(frt):
     g = torch.Generator().manual_seed(1)
     a = torch.randn(777, 640, generator=g).to(torch.bfloat16).cuda()
