@@ -198,17 +198,19 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 }
                 const CUtensorMap* map = (L & 1) ? &sd.v_map : &sd.k_map;
                 const int row = (t0 + (L >> 1)) * kBN;
-                const uint32_t fb = smem_u32(&bars->kv_full[stage]);
-                mbar_arrive_expect_tx(fb, C::KV_TILE);
+                // K_j and V_j (loads 2j, 2j+1) complete on one barrier, kv_full[j % 4]:
+                // the MMA thread then tests one barrier per KV step instead of two
+                const uint32_t fb = smem_u32(&bars->kv_full[(L >> 1) & 3]);
+                if ((L & 1) == 0) mbar_arrive_expect_tx(fb, 2 * C::KV_TILE);
                 const uint32_t dst = sKV + stage * C::KV_TILE;
                 for (int cb = 0; cb < C::NCB; ++cb)
                     tma_load_3d(dst + cb * (kBN * 128), map, fb, cb * 64, head, row);
             }
-            // drain: every issued load must have landed before the CTA may exit
-            const int first = (L - C::STAGES) > 0 ? (L - C::STAGES) : 0;
-            for (int Ld = first; Ld < L; ++Ld)
-                mbar_wait_drain(smem_u32(&bars->kv_full[Ld % C::STAGES]), (Ld / C::STAGES) & 1,
-                                lim);
+            // drain: every issued load must have landed before the CTA may exit (a pair
+            // left half-issued by an error completes only by the wait's time limit)
+            const int npairs = (L + 1) >> 1;
+            for (int pr = (npairs > 4 ? npairs - 4 : 0); pr < npairs; ++pr)
+                mbar_wait_drain(smem_u32(&bars->kv_full[pr & 3]), (pr >> 2) & 1, lim);
             mbar_wait_drain(qbar, 0, lim);
         }
       } else if (warp == 1) {
@@ -228,9 +230,14 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             const uint64_t dq0 = sdesc_sw128(sQ, 16, 1024);
             const uint64_t dk0 = sdesc_sw128(sKV, 16, 1024);
             const uint64_t dv0 = sdesc_sw128(sKV, kBN * 128, 1024);
+            // K_j and V_j share a barrier, kv_full[j % 4]: waiting for K_j (load 2j)
+            // covers V_j, so the wait for load 2j+1 is a no-op. Pair j+4 is loaded only
+            // after step j-1's slot release, which this thread commits after it waited
+            // for pair j, so the parity of kv_full[j % 4] is never ambiguous.
             auto wait_load = [&](int Lw) -> bool {
-                const uint32_t fb = smem_u32(&bars->kv_full[Lw % C::STAGES]);
-                const uint32_t par = (Lw / C::STAGES) & 1;
+                if (Lw & 1) return true;
+                const uint32_t fb = smem_u32(&bars->kv_full[(Lw >> 1) & 3]);
+                const uint32_t par = ((Lw >> 1) >> 2) & 1;
                 if (!mbar_test_wait(fb, par) && !mbar_wait(fb, par, lim, abort)) {
                     report(p.status, abort, 1, Lw);
                     return false;
