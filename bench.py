@@ -471,16 +471,16 @@ def run_gpu_conv(args, cw, world, rank, local):
                                f"{cw.kt}x{cw.kh}x{cw.kw} (causal in time, cache of "
                                f"{cw.kt - 1} frames), {cw.grid_h}x{cw.grid_w} pixels, "
                                f"{cw.frames} frames/chunk",
-                   "path": "frt_conv_step (implicit GEMM on tcgen05 + cache update: 2 launches)",
+                   "path": "frt_conv_step (implicit GEMM on tcgen05 with the cache update fused: 1 launch)",
                    "l2": f"{POOL} distinct chunks of {x_bytes / 1e6:.1f} MB cycled",
                    "flops_per_step": flops},
         "roofline": {"bound": "tensor", "achieved": round(flops / (step_ms * 1e-3) / 1e12, 2),
                      "peak": peak_tf, "unit": "TFLOP/s",
                      "frac": round(flops / (step_ms * 1e-3) / 1e12 / peak_tf, 4), "traffic": None,
-                     "kernel": "conv_kernel (+ cache_shift_kernel)", "peak_kind": peak_kind,
+                     "kernel": "conv_kernel (cache update fused)", "peak_kind": peak_kind,
                      "launch_ms": round(step_ms, 4)},
         "clocks": clk.summary(),
-        "gpu_launches": (2 if cw.kt > 1 else 1) * n,
+        "gpu_launches": n,
     }
 
 

@@ -193,7 +193,8 @@ frt_conv_t* frt_conv_create(int cin, int cout, int kt, int kh, int kw, int grid_
  * cudaStream_t every later call enqueues on. May be called again to change them. */
 frt_status frt_conv_configure(frt_conv_t* c, int out_dtype, void* cuda_stream);
 /* One chunk: y from (cache, x), then the cache becomes the last kt - 1 frames of
- * (cache, x). Two launches (the convolution on the tensor cores, the cache update). */
+ * (cache, x). One launch (the convolution on the tensor cores; its epilogue warps write
+ * the next cache into the other half of a ping-pong pair while the MMAs run). */
 frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w,
                          const void* bias, void* y);
 /* Tile of the convolution kernel, for tuning and tests (no counterpart in the paper):

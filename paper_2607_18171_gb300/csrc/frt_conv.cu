@@ -33,8 +33,9 @@
 // CTAs of a cluster work as a pair on two pixel tiles with tcgen05.mma.cta_group::2 (M =
 // 256): each holds its own halo and half of the weight slice, which halves the weight
 // bytes each SM takes in per FLOP — with the halo, the larger share of what bounds this
-// kernel. A second, small kernel writes the next cache (last kt - 1 frames of (cache,
-// chunk)) into the other half of a ping-pong pair, so no launch reads what it writes.
+// kernel. The next cache (last kt - 1 frames of (cache, chunk)) is written into the other
+// half of a ping-pong pair by the epilogue warps of every CTA, a slice each, while they
+// wait for their first accumulator; no launch reads what it writes.
 #include <algorithm>
 #include <cstring>
 #include <mutex>
@@ -75,6 +76,13 @@ struct ConvParams {
     int b_stage;            // weight-ring stage bytes: tb * (BN / pair) * 128
     unsigned long long wait_limit_ns;
     DeviceStatus* status;
+    // next cache = frames [F, F + keep) of (cache, chunk), in 16-byte vectors (keep = 0:
+    // no cache)
+    const uint4* shift_cache;
+    const uint4* shift_x;
+    uint4* shift_next;
+    long long shift_frame_vec;   // vectors per frame
+    int shift_keep;              // kt - 1
 };
 
 template <int BN, bool PAIR>
@@ -369,6 +377,21 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
         const uint32_t sw = uint32_t(row & 7);
         const bool est = threadIdx.x == 64;              // issues the tile's TMA stores
         const int ucols = p.y_bf16 ? 64 : 32;            // output channels per unit
+        if (p.shift_keep > 0) {
+            // this CTA's slice of the next cache, while the first tile's MMAs run
+            const long long total = p.shift_frame_vec * p.shift_keep;
+            const long long per = (total + gridDim.x - 1) / gridDim.x;
+            const long long lo = per * blockIdx.x;
+            const long long hi = lo + per < total ? lo + per : total;
+            for (long long i = lo + (threadIdx.x - 64); i < hi; i += 128) {
+                const int j = int(i / p.shift_frame_vec);
+                const long long r = i - (long long)j * p.shift_frame_vec;
+                const int src = j + p.F;                     // frame of (cache, chunk)
+                p.shift_next[i] = src < p.shift_keep
+                                      ? __ldg(p.shift_cache + (long long)src * p.shift_frame_vec + r)
+                                      : __ldg(p.shift_x + (long long)(src - p.shift_keep) * p.shift_frame_vec + r);
+            }
+        }
         int tl = 0;
         for (int t = c_first; t < p.n_tiles; t += c_stride, ++tl) {
             const int b = tl & 1;
@@ -438,20 +461,6 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     if (warp == 1) {
         if (PAIR) tmem_dealloc_pair(tmem, C::TMEM_COLS);
         else tmem_dealloc(tmem, C::TMEM_COLS);
-    }
-}
-
-// next cache = last kt - 1 frames of (cache, chunk), written to the other ping-pong half
-__global__ void cache_shift_kernel(const uint4* __restrict__ cache, const uint4* __restrict__ x,
-                                   uint4* __restrict__ next, long long frame_vec, int keep, int F) {
-    const long long total = frame_vec * keep;
-    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
-         i += (long long)gridDim.x * blockDim.x) {
-        const int j = int(i / frame_vec);          // frame of the next cache
-        const long long r = i - (long long)j * frame_vec;
-        const int src = j + F;                     // frame of (cache, chunk)
-        next[i] = src < keep ? cache[(long long)src * frame_vec + r]
-                             : x[(long long)(src - keep) * frame_vec + r];
     }
 }
 
@@ -733,6 +742,13 @@ frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w, const void
     p.y_bf16 = c->out_dtype == FRT_OUT_BF16;
     p.wait_limit_ns = c->wait_limit_ns;
     p.status = c->status_dev;
+    if (c->kt > 1) {
+        p.shift_cache = static_cast<const uint4*>(c->cache[c->cur]);
+        p.shift_x = static_cast<const uint4*>(x);
+        p.shift_next = static_cast<uint4*>(c->cache[c->cur ^ 1]);
+        p.shift_frame_vec = (long long)(c->frame_bytes / 16);
+        p.shift_keep = c->kt - 1;
+    }
     cudaError_t e;
     switch (bn * 2 + (pair ? 1 : 0)) {
         case 513: e = launch_conv<256, true>(p, c->cs); break;
@@ -747,19 +763,7 @@ frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w, const void
         default: e = launch_conv<64, false>(p, c->cs); break;
     }
     if (e != cudaSuccess) return cfail(FRT_ERR_CUDA, cudaGetErrorString(e));
-    if (c->kt > 1) {
-        const int keep = c->kt - 1;
-        const long long frame_vec = (long long)(c->frame_bytes / 16);
-        const long long total = frame_vec * keep;
-        const int blocks = int(std::min<long long>((total + 255) / 256, 4LL * num_sms()));
-        cache_shift_kernel<<<blocks, 256, 0, c->cs>>>(static_cast<const uint4*>(c->cache[c->cur]),
-                                                       static_cast<const uint4*>(x),
-                                                       static_cast<uint4*>(c->cache[c->cur ^ 1]),
-                                                       frame_vec, keep, c->F);
-        if ((e = cudaGetLastError()) != cudaSuccess)
-            return cfail(FRT_ERR_CUDA, cudaGetErrorString(e));
-        c->cur ^= 1;
-    }
+    if (c->kt > 1) c->cur ^= 1;
     c->chunks += 1;
     return FRT_OK;
 }
