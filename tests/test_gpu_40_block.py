@@ -82,6 +82,26 @@ def test_gemm_every_tile_width_matches_fp64(frt, M, N, K, bn):
     assert np.all(err <= bound + 1e-30), f"bn {bn}: max excess {float(np.max(err - bound)):.3e}"
 
 
+def test_gemm_tile_width_does_not_change_results(frt):
+    """Each output sums its products in one order (k-block, 16-deep step) whatever the
+    tile width: every width gives the same bits."""
+    g = torch.Generator().manual_seed(3)
+    a = torch.randn(1000, 1536, generator=g).to(torch.bfloat16).cuda()
+    b = torch.randn(960, 1536, generator=g).to(torch.bfloat16).cuda()
+    outs = []
+    try:
+        for bn in (128, 192, 256):
+            frt.selftest_gemm_force_bn(bn)
+            c = torch.empty(1000, 960, device="cuda")
+            frt.gemm_bf16(a, b, c)
+            outs.append(c)
+        torch.cuda.synchronize()
+    finally:
+        frt.selftest_gemm_force_bn(0)
+    for c in outs[1:]:
+        assert torch.equal(outs[0], c)
+
+
 def test_gemm_is_deterministic(frt):
     g = torch.Generator().manual_seed(1)
     a = torch.randn(777, 640, generator=g).to(torch.bfloat16).cuda()
