@@ -439,7 +439,10 @@ int gemm_cluster_m(int M) { return M > kBM ? 2 : 1; }
 
 // Output columns per tile: the width in {128, 192, 256} with the least rounds of tiles
 // over the SMs (or SM pairs) x width, a 128-wide tile weighted 1.5x (measured: an N = 128
-// MMA of a CTA pair issues in ~82 cycles for 64 of work and its stage waits are exposed).
+// MMA of a CTA pair issues in ~82 cycles for 64 of work and its stage waits are exposed)
+// and a 192-wide one 1.15x (measured per round and column against 256-wide tiles: 1.14x
+// on a 4680 x 4608 x 1536 projection, 1.21x on 4680 x 1536 x 1536; each A k-block feeds
+// fewer columns, so more operand bytes cross into the SMs per FLOP).
 // The QKV epilogue needs a width dividing d (a tile never straddles q, k and v); widths
 // past N are not considered unless nothing else fits.
 int g_force_bn = 0;   // test override (frt_selftest_gemm_force_bn)
@@ -455,7 +458,7 @@ int gemm_block_n_for(int M, int N, int epi, int d) {
         if (epi == kEpiQkv && d % bn != 0) continue;
         if (bn > 128 && bn > N) continue;
         const long long tiles = ctm * ((N + bn - 1) / bn);
-        const double t = double((tiles + units - 1) / units) * bn * (bn == 128 ? 1.5 : 1.0);
+        const double t = double((tiles + units - 1) / units) * bn * (bn == 128 ? 1.5 : (bn == 192 ? 1.15 : 1.0));
         if (t < best_t - 1e-9) {
             best_t = t;
             best = bn;
