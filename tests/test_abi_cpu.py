@@ -70,6 +70,16 @@ def test_create_validates_shapes(frt):
     h = L.frt_stream_create(2, 64, 16, 3, 3)
     assert h
     L.frt_stream_destroy(h)
+    # the limits themselves: heads * head_dim <= 12800, Nq <= 2^20, W * Nq <= 2^24
+    for args, ok in (((100, 128, 16, 3, 3), True), ((101, 128, 16, 3, 3), False),
+                     ((200, 64, 16, 3, 3), True), ((201, 64, 16, 3, 3), False),
+                     ((1, 64, 1, 1, 1), True),
+                     ((1, 64, 1 << 20, 1, 16), True), ((1, 64, 1 << 20, 1, 17), False),
+                     ((1, 64, (1 << 20) + 1, 1, 1), False)):
+        h = L.frt_stream_create(*args)
+        assert bool(h) == ok, args
+        if h:
+            L.frt_stream_destroy(h)
 
 
 def test_configure_rejects_bad_config_before_device_work(frt):

@@ -28,6 +28,10 @@ SMALL = {
     "d64_multi_tile": synth.Workload("d64_multi_tile", 92, 1, 3, 64, 8, 10, 2, 2, 4, (16, 24, 24)),
     # window 1: plain bidirectional attention per chunk
     "window1": synth.Workload("window1", 93, 1, 2, 128, 5, 9, 2, 1, 3, (32, 48, 48)),
+    # the widest token row the library accepts: heads * head_dim = 12800 (25.6 KB rows)
+    "max_row": synth.Workload("max_row", 94, 1, 100, 128, 4, 5, 2, 2, 3, (32, 48, 48)),
+    # the smallest chunk: one token (1 x 1 grid, one frame); Nkv 1..3, far below one tile
+    "one_token": synth.Workload("one_token", 95, 1, 2, 64, 1, 1, 1, 3, 5, (16, 24, 24)),
 }
 
 
