@@ -126,6 +126,16 @@ def test_product_path_does_not_import_the_oracle():
                 assert not re.search(r"^\s*(import|from)\s+oracle", src, flags=re.M), f
 
 
+def test_batched_rejects_stream_counts_outside_1_to_32(frt):
+    L = frt.lib()
+    bad = L.frt_chunk_attention_batched.argtypes[0]._type_
+    arr = (bad * 33)()
+    for n in (0, -1, 33):
+        assert L.frt_chunk_attention_batched(arr, n, arr, arr) == 1, n   # FRT_ERR_INVALID_ARG
+        assert "1 <= n <= 32" in L.frt_last_error().decode()
+    assert L.frt_chunk_attention_batched(None, 1, arr, arr) == 1
+
+
 def test_step_group_argument_checks(frt):
     L = frt.lib()
     assert not L.frt_steps_create(0, 2, 64, 16, 3, 3)

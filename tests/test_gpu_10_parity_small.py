@@ -164,6 +164,31 @@ def test_batched_ragged_streams_match_single_launches_and_oracle(frt):
         st.close()
 
 
+def test_batched_at_the_stream_limit(frt):
+    """32 streams, the most one batched launch takes, with fills 1..W, against the oracle."""
+    base = synth.WORKLOADS["tiny"]
+    fills = [1 + s % base.window for s in range(32)]
+    streams, qs, outs = [], [], []
+    for s, fill in enumerate(fills):
+        st = U.make_stream(base, frt)
+        for c in range(fill - 1):
+            q, k, v = U.gpu_inputs(base, s, c)
+            st.chunk_step(q, k, v, st.new_out())
+        q, k, v = U.gpu_inputs(base, s, fill - 1)
+        st.rope3d_qk(q, k)
+        st.kv_append_evict(k, v)
+        streams.append(st)
+        qs.append(q)
+        outs.append(st.new_out())
+    frt.chunk_attention_batched(streams, qs, outs)
+    torch.cuda.synchronize()
+    for s, fill in enumerate(fills):
+        ref = U.oracle_full_stream(base, s, fill)[fill - 1][0]
+        U.assert_close(outs[s].cpu().numpy(), ref, f"stream {s}")
+    for st in streams:
+        st.close()
+
+
 def test_host_buffer_step_pipelined_matches_device_path_and_oracle(frt):
     """frt_chunk_step_host keeps several chunks in flight (copy-in, compute and
     copy-out overlap across calls); after one sync every chunk's output must equal

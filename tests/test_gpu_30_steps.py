@@ -20,7 +20,7 @@ def frt():
     return m
 
 
-@pytest.mark.parametrize("n_steps,window,chunks", [(3, 3, 5), (4, 2, 3)])
+@pytest.mark.parametrize("n_steps,window,chunks", [(3, 3, 5), (4, 2, 3), (32, 2, 2)])
 def test_wavefront_ticks_match_per_step_oracles(frt, n_steps, window, chunks):
     base = synth.Workload("steps", 96, 1, 3, 128, 10, 13, 3, window, chunks, (32, 48, 48))
     grp = frt.Steps(n_steps, base.heads, base.head_dim, base.grid_h, base.grid_w, base.frames,
