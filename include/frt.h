@@ -78,7 +78,9 @@ frt_status frt_config_default(const frt_stream_t* s, frt_config* cfg);
 
 /* Validate and apply *cfg; allocates (once) and zero-fills the KV cache
  * (2 * window_chunks * Nq * heads * head_dim bf16) and the RoPE tables, and
- * resets the chunk counter to 0. Synchronous. Must precede every other call. */
+ * resets the chunk counter to 0. Synchronous. Must precede every other call.
+ * A configure that fails after validation leaves the stream unconfigured: later
+ * calls return FRT_ERR_STATE until a configure succeeds. */
 frt_status frt_stream_configure(frt_stream_t* s, const frt_config* cfg);
 
 /* Operation 1: rotate q and k (bf16 [Nq, heads, head_dim]) in place at the
@@ -279,7 +281,8 @@ void frt_steps_destroy(frt_steps_t* g);
  * first device error, e.g. FRT_ERR_TIMEOUT). */
 frt_status frt_stream_sync(frt_stream_t* s);
 
-/* Clear the cache contents, chunk counter, ordering state and device status. */
+/* Clear the cache contents, chunk counter, ordering state, split-KV merge
+ * counters and device status (the way back after FRT_ERR_TIMEOUT). */
 frt_status frt_stream_reset(frt_stream_t* s);
 
 /* Release everything the handle owns (waits for its work first). NULL is a no-op. */

@@ -614,6 +614,11 @@ frt_status cfail(frt_status st, const char* msg) {
     set_last_error(msg);
     return st;
 }
+// A CUDA runtime call of this layer failed (see clear_cuda_error).
+frt_status cuda_cfail(frt_status st, const char* msg) {
+    clear_cuda_error();
+    return cfail(st, msg);
+}
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 void free_conv(frt_conv_t* c) {
     for (int i = 0; i < 2; ++i)
@@ -662,18 +667,18 @@ frt_status frt_conv_configure(frt_conv_t* c, int out_dtype, void* cuda_stream) {
             if ((e = cudaMalloc(&c->cache[i], bytes)) != cudaSuccess ||
                 (e = cudaMemset(c->cache[i], 0, bytes)) != cudaSuccess) {
                 free_conv(c);
-                return cfail(e == cudaErrorMemoryAllocation ? FRT_ERR_OOM : FRT_ERR_CUDA,
-                             "frame cache allocation failed");
+                return cuda_cfail(e == cudaErrorMemoryAllocation ? FRT_ERR_OOM : FRT_ERR_CUDA,
+                                  "frame cache allocation failed");
             }
         if ((e = cudaHostAlloc(reinterpret_cast<void**>(&c->status_host), sizeof(DeviceStatus),
                                cudaHostAllocMapped)) != cudaSuccess ||
             (e = cudaHostGetDevicePointer(reinterpret_cast<void**>(&c->status_dev), c->status_host,
                                           0)) != cudaSuccess) {
             free_conv(c);
-            return cfail(FRT_ERR_CUDA, "status allocation failed");
+            return cuda_cfail(FRT_ERR_CUDA, "status allocation failed");
         }
         std::memset(c->status_host, 0, sizeof(DeviceStatus));
-        if ((e = cudaDeviceSynchronize()) != cudaSuccess) return cfail(FRT_ERR_CUDA, "sync failed");
+        if ((e = cudaDeviceSynchronize()) != cudaSuccess) return cuda_cfail(FRT_ERR_CUDA, "sync failed");
     }
     c->out_dtype = out_dtype;
     c->cs = static_cast<cudaStream_t>(cuda_stream);
@@ -762,7 +767,7 @@ frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w, const void
         case 129: e = launch_conv<64, true>(p, c->cs); break;
         default: e = launch_conv<64, false>(p, c->cs); break;
     }
-    if (e != cudaSuccess) return cfail(FRT_ERR_CUDA, cudaGetErrorString(e));
+    if (e != cudaSuccess) return cuda_cfail(FRT_ERR_CUDA, cudaGetErrorString(e));
     if (c->kt > 1) c->cur ^= 1;
     c->chunks += 1;
     return FRT_OK;
@@ -794,7 +799,7 @@ frt_status frt_conv_sync(frt_conv_t* c) {
     if (!c) return cfail(FRT_ERR_INVALID_ARG, "NULL conv handle");
     if (!c->configured) return FRT_OK;
     cudaError_t e = cudaStreamSynchronize(c->cs);
-    if (e != cudaSuccess) return cfail(FRT_ERR_CUDA, cudaGetErrorString(e));
+    if (e != cudaSuccess) return cuda_cfail(FRT_ERR_CUDA, cudaGetErrorString(e));
     if (c->status_host && c->status_host->code != 0)
         return cfail(static_cast<frt_status>(c->status_host->code),
                      "a device-side bounded wait gave up");
@@ -807,7 +812,7 @@ frt_status frt_conv_reset(frt_conv_t* c) {
     cudaError_t e = cudaStreamSynchronize(c->cs);
     const size_t bytes = std::max<size_t>(1, size_t(c->kt - 1)) * c->frame_bytes;
     for (int i = 0; i < 2 && e == cudaSuccess; ++i) e = cudaMemset(c->cache[i], 0, bytes);
-    if (e != cudaSuccess) return cfail(FRT_ERR_CUDA, cudaGetErrorString(e));
+    if (e != cudaSuccess) return cuda_cfail(FRT_ERR_CUDA, cudaGetErrorString(e));
     std::memset(c->status_host, 0, sizeof(DeviceStatus));
     c->cur = 0;
     c->chunks = 0;

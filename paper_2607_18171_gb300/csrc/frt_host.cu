@@ -33,6 +33,7 @@ frt_status fail(frt_status st, const char* fmt, ...) {
 }
 
 frt_status cuda_fail(cudaError_t e, const char* what) {
+    clear_cuda_error();
     return fail(e == cudaErrorMemoryAllocation ? FRT_ERR_OOM : FRT_ERR_CUDA, "%s: %s", what,
                 cudaGetErrorString(e));
 }
@@ -534,6 +535,9 @@ frt_status frt_stream_configure(frt_stream_t* s, const frt_config* cfg) {
         cudaError_t e = cudaStreamSynchronize(s->cs);
         if (e != cudaSuccess) return cuda_fail(e, "sync before reconfigure");
     }
+    // a configure that fails part-way leaves the stream unconfigured, never half-built:
+    // later calls return FRT_ERR_STATE until a configure succeeds
+    s->configured = false;
     s->cfg = *cfg;
     s->scale = float(cfg->sm_scale > 0 ? cfg->sm_scale : 1.0 / std::sqrt(double(s->head_dim)));
     s->cs = static_cast<cudaStream_t>(cfg->cuda_stream);
@@ -595,9 +599,12 @@ frt_status frt_stream_configure(frt_stream_t* s, const frt_config* cfg) {
             return st;
         }
     }
-    // zero cache: rows past the valid prefix are never read by value, but keep them finite
+    // zero cache: rows past the valid prefix are never read by value, but keep them finite;
+    // zero merge counters: a launch that gave up part-way may have left some counted
     if ((e = cudaMemset(s->cache_k, 0, cache_bytes)) != cudaSuccess ||
-        (e = cudaMemset(s->cache_v, 0, cache_bytes)) != cudaSuccess)
+        (e = cudaMemset(s->cache_v, 0, cache_bytes)) != cudaSuccess ||
+        (s->counters &&
+         (e = cudaMemset(s->counters, 0, size_t(s->part_groups) * sizeof(int))) != cudaSuccess))
         return cuda_fail(e, "cache clear");
     if ((e = cudaDeviceSynchronize()) != cudaSuccess) return cuda_fail(e, "configure sync");
     s->counter = 0;
@@ -973,8 +980,12 @@ frt_status frt_stream_reset(frt_stream_t* s) {
     if (e == cudaSuccess && s->cp_out) e = cudaStreamSynchronize(s->cp_out);
     if (e != cudaSuccess) return cuda_fail(e, "stream sync");
     const size_t cache_bytes = size_t(s->window) * s->chunk_elems * 2;
+    // the merge counters too: a launch that gave up part-way (the usual reason for a
+    // reset) may have left some of them counted, which would elect a merging split early
     if ((e = cudaMemsetAsync(s->cache_k, 0, cache_bytes, s->cs)) != cudaSuccess ||
         (e = cudaMemsetAsync(s->cache_v, 0, cache_bytes, s->cs)) != cudaSuccess ||
+        (s->counters && (e = cudaMemsetAsync(s->counters, 0, size_t(s->part_groups) * sizeof(int),
+                                             s->cs)) != cudaSuccess) ||
         (e = cudaStreamSynchronize(s->cs)) != cudaSuccess)
         return cuda_fail(e, "cache clear");
     std::memset(s->status_host, 0, sizeof(DeviceStatus));
@@ -986,7 +997,8 @@ frt_status frt_stream_reset(frt_stream_t* s) {
 
 void frt_stream_destroy(frt_stream_t* s) {
     if (!s) return;
-    if (s->configured) cudaStreamSynchronize(s->cs);
+    // device memory may exist without a completed configure (one that failed part-way)
+    if (s->configured || s->cache_k || s->stage) cudaStreamSynchronize(s->cs);
     free_device(s);
     delete s;
 }

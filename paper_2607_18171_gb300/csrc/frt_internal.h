@@ -178,5 +178,9 @@ cudaError_t launch_attention_batched(const AttnParams<kMaxBatchStreams>& p, int 
 int num_sms();
 // Set the thread-local message that frt_last_error() returns.
 void set_last_error(const char* msg);
+// Report a CUDA runtime call of the library that failed: the message is kept for
+// frt_last_error() and the runtime's (non-sticky) last error is cleared, so that it does
+// not surface again from the caller's next, unrelated CUDA call.
+inline void clear_cuda_error() { (void)cudaGetLastError(); }
 
 }  // namespace frt

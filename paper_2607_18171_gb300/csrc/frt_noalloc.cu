@@ -98,6 +98,11 @@ frt_status fail(frt_status st, const char* msg) {
     set_last_error(msg);
     return st;
 }
+// A CUDA runtime call of this entry point failed (see clear_cuda_error).
+frt_status cuda_failed(const char* msg) {
+    clear_cuda_error();
+    return fail(FRT_ERR_CUDA, msg);
+}
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -128,7 +133,7 @@ extern "C" frt_status frt_chunk_attention_noalloc(const void* q, const void* k, 
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess || dev < 0 || dev >= kMaxDevices)
-        return fail(FRT_ERR_CUDA, "no usable current device");
+        return cuda_failed("no usable current device");
     void* base = nullptr;
     {
         std::lock_guard<std::mutex> lock(g_mu);
@@ -136,7 +141,7 @@ extern "C" frt_status frt_chunk_attention_noalloc(const void* q, const void* k, 
             void* ptr = nullptr;
             e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
             if (e != cudaSuccess || !ptr)
-                return fail(FRT_ERR_CUDA, "cudaGetSymbolAddress of the static scratch failed");
+                return cuda_failed("cudaGetSymbolAddress of the static scratch failed");
             g_scratch_dev[dev] = ptr;
         }
         base = g_scratch_dev[dev];
@@ -190,8 +195,8 @@ extern "C" frt_status frt_chunk_attention_noalloc(const void* q, const void* k, 
     // merge counters must start at zero: clear this call's share of the shared array
     if (split > 1 &&
         (e = cudaMemsetAsync(counters, 0, size_t(groups) * sizeof(int), st)) != cudaSuccess)
-        return fail(FRT_ERR_CUDA, "clearing the merge counters failed");
+        return cuda_failed("clearing the merge counters failed");
     if ((e = launch_attention_single(p, head_dim, false, st)) != cudaSuccess)
-        return fail(FRT_ERR_CUDA, cudaGetErrorString(e));
+        return cuda_failed(cudaGetErrorString(e));
     return FRT_OK;
 }

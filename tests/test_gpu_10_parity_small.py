@@ -78,6 +78,41 @@ def test_run_to_run_determinism(frt):
         assert np.array_equal(outs[0][c][0], outs[1][c][0])
 
 
+def test_reset_restarts_the_stream_bit_identically(frt):
+    """After reset (cache, counter, split-KV merge counters, status cleared) a stream
+    reproduces a fresh stream's outputs bit for bit."""
+    wl = SMALL["ragged_d128"]
+    fresh = U.make_stream(wl, frt)
+    ref = U.run_fused(fresh, wl, 0, wl.chunks, keep=range(wl.chunks))
+    fresh.close()
+    st = U.make_stream(wl, frt)
+    U.run_fused(st, wl, 1, 2)            # other inputs first
+    st.reset()
+    got = U.run_fused(st, wl, 0, wl.chunks, keep=range(wl.chunks))
+    for c in range(wl.chunks):
+        assert got[c][1:] == ref[c][1:]
+        assert np.array_equal(got[c][0], ref[c][0]), f"chunk {c}"
+    st.close()
+
+
+def test_failed_configure_leaves_the_stream_unconfigured(frt):
+    import ctypes
+    L = frt.lib()
+    # accepted shape (Nq = 2^20, W * Nq = 2^24, heads * head_dim = 12800) whose cache,
+    # 2 x 430 GB, no GPU holds: the allocation fails cleanly with FRT_ERR_OOM
+    h = L.frt_stream_create(100, 128, 1 << 16, 16, 16)
+    assert h
+    cfg = frt.Config()
+    assert L.frt_config_default(h, ctypes.byref(cfg)) == 0
+    assert L.frt_stream_configure(h, ctypes.byref(cfg)) == 3          # FRT_ERR_OOM
+    buf = ctypes.create_string_buffer(64)
+    p = ctypes.cast(buf, ctypes.c_void_p)
+    assert L.frt_rope3d_qk(h, p, p) == 2                              # FRT_ERR_STATE
+    assert L.frt_stream_reset(h) == 2
+    L.frt_stream_destroy(h)
+    torch.cuda.synchronize()                                         # the context is fine
+
+
 def test_bf16_output(frt):
     wl = SMALL["ragged_d128"]
     st = U.make_stream(wl, frt, out_dtype=torch.bfloat16)
