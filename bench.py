@@ -42,6 +42,12 @@ def describe(wl) -> str:
             f"window {wl.window} chunks (Nkv {wl.window * wl.n_q} at steady state)")
 
 
+def describe_conv(cw) -> str:
+    return (f"{cw.name}: Cin {cw.cin}, Cout {cw.cout}, kernel {cw.kt}x{cw.kh}x{cw.kw} "
+            f"(causal in time, cache of {cw.kt - 1} frames), {cw.grid_h}x{cw.grid_w} pixels, "
+            f"{cw.frames} frames/chunk")
+
+
 def load_peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -467,10 +473,7 @@ def run_gpu_conv(args, cw, world, rank, local):
         "ms_per_step": round(elapsed / n, 4), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded N(0,1) channels-last frames, N(0,1/(taps*Cin)) weights)",
-        "config": {"workload": f"{cw.name}: Cin {cw.cin}, Cout {cw.cout}, kernel "
-                               f"{cw.kt}x{cw.kh}x{cw.kw} (causal in time, cache of "
-                               f"{cw.kt - 1} frames), {cw.grid_h}x{cw.grid_w} pixels, "
-                               f"{cw.frames} frames/chunk",
+        "config": {"workload": describe_conv(cw),
                    "path": "frt_conv_step (implicit GEMM on tcgen05 with the cache update fused: 1 launch)",
                    "l2": f"{POOL} distinct chunks of {x_bytes / 1e6:.1f} MB cycled",
                    "flops_per_step": flops},
@@ -655,6 +658,18 @@ def cpu_baseline(wl, seconds: float = 15.0):
                       f"{wl.heads} heads ({dt:.1f} s)"}
 
 
+def _reference_line(args, world, metric, value, total, n, config, sample):
+    return {"metric": metric, "value": round(value, 6), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(1e3 * total / n, 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "impl": "reference", "config": config,
+            "cpu_baseline": {"value": round(value, 6), "unit": UNIT, "cores": cpu_threads(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(value, 6), "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
 def run_reference(args, wl, world, rank):
     """Reference arm: the oracle timed as it stands on the host cores, one bounded
     sample of the workload per step (one head, a row subset sized so the whole run
@@ -675,19 +690,91 @@ def run_reference(args, wl, world, rank):
             times.append(t)
     total = sum(times)
     flops = 4 * len(rows) * nkv * wl.head_dim * heads
-    value = flops * len(times) / total / 1e12
-    sample = (f"per step: one full-window chunk of {wl.name} (RoPE of the chunk, append, "
-              f"exact fp64 attention) for {len(rows)} of {wl.n_q} query rows x {heads} of "
-              f"{wl.heads} heads")
-    return {"metric": METRIC, "value": round(value, 6), "unit": UNIT, "n_gpus": world,
-            "steps": args.steps, "warmup": args.warmup,
-            "ms_per_step": round(1e3 * total / len(times), 3), "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "impl": "reference", "config": {"workload": describe(wl)},
-            "cpu_baseline": {"value": round(value, 6), "unit": UNIT, "cores": cpu_threads(),
-                             "kind": "oracle", "sample": sample},
-            "e2e": {"value": round(value, 6), "unit": UNIT, "h2d_bytes_per_step": 0,
-                    "d2h_bytes_per_step": 0}}
+    return _reference_line(
+        args, world, METRIC, flops * len(times) / total / 1e12, total, len(times),
+        {"workload": describe(wl)},
+        f"per step: one full-window chunk of {wl.name} (RoPE of the chunk, append, exact "
+        f"fp64 attention) for {len(rows)} of {wl.n_q} query rows x {heads} of {wl.heads} heads")
+
+
+def run_reference_conv(args, cw, world, rank):
+    """Reference arm of a convolution workload: the oracle's streaming convolution as it
+    stands, one chunk per step for a subset of the output channels (each output channel
+    is computed independently of the others), sized so the run fits --ref-seconds."""
+    if rank != 0:
+        return None
+    from oracle.frt_oracle import OracleConvStream
+    from paper_2607_18171_gb300 import synth
+    w, b = synth.conv_weights(cw)
+    w64, b64 = synth.as_f64(w), np.asarray(b, np.float64)
+    orc = OracleConvStream(cw.cin, cw.cout, cw.kt, cw.kh, cw.kw, cw.grid_h, cw.grid_w)
+    probe = min(cw.cout, 32)
+    t = time.perf_counter()
+    orc.step(synth.as_f64(synth.conv_chunk(cw, 0, 0)), w64[:, :probe], b64[:probe])
+    dt = time.perf_counter() - t
+    per_step = args.ref_seconds / max(1, args.steps + args.warmup)
+    n_c = max(1, min(cw.cout, int(probe * per_step / max(dt, 1e-3))))
+    times = []
+    for i in range(args.warmup + args.steps):
+        x = synth.as_f64(synth.conv_chunk(cw, 0, 1 + i))
+        t = time.perf_counter()
+        orc.step(x, w64[:, :n_c], b64[:n_c])
+        if i >= args.warmup:
+            times.append(time.perf_counter() - t)
+    total = sum(times)
+    flops = 2 * cw.frames * cw.grid_h * cw.grid_w * n_c * cw.taps * cw.cin
+    return _reference_line(
+        args, world, CONV_METRIC, flops * len(times) / total / 1e12, total, len(times),
+        {"workload": describe_conv(cw)},
+        f"per step: one chunk of {cw.name} through the oracle's streaming convolution for "
+        f"{n_c} of {cw.cout} output channels")
+
+
+def run_reference_block(args, wl, world, rank):
+    """Reference arm of the DiT-block slice: the oracle's pieces as they stand (linear,
+    the chunk step, linear) on one head's share of the block per step — that head's q, k,
+    v projection columns for every token (the cache needs k and v of every token), RoPE,
+    append and attention for a subset of query rows, and that head's share of the output
+    projection for those rows. Heads are independent up to the output projection, whose
+    head shares add up."""
+    if rank != 0:
+        return None
+    from oracle.frt_oracle import OracleStream, bf16_round, linear
+    from paper_2607_18171_gb300 import synth
+    d, D = wl.heads * wl.head_dim, wl.head_dim
+    w_qkv, w_o = (synth.as_f64(t) for t in synth.block_weights(wl))
+    w_h = np.concatenate([w_qkv[i * d:i * d + D] for i in range(3)])   # head 0's rows
+    w_oh = w_o[:, :D]
+    orc = OracleStream(1, D, wl.grid_h, wl.grid_w, wl.frames, wl.window, wl.split)
+
+    def step(chunk, rows):
+        x = synth.as_f64(synth.chunk_x(wl, 0, chunk))
+        t = time.perf_counter()
+        qkv = bf16_round(linear(x, w_h))
+        q, k, v = (qkv[:, i * D:(i + 1) * D].reshape(wl.n_q, 1, D) for i in range(3))
+        o, _, _ = orc.step(q, k, v, rows=rows)
+        linear(bf16_round(o).reshape(len(rows), D), w_oh)
+        return time.perf_counter() - t
+
+    probe = _rows_for(wl.n_q, 16)
+    for c in range(wl.window - 1):
+        dt = step(c, probe)
+    per_step = args.ref_seconds / max(1, args.steps + args.warmup)
+    rows = _rows_for(wl.n_q, len(probe) * per_step / max(dt, 1e-3))
+    times = []
+    for i in range(args.warmup + args.steps):
+        t = step(wl.window - 1 + i, rows)
+        if i >= args.warmup:
+            times.append(t)
+    total = sum(times)
+    nkv = wl.window * wl.n_q
+    flops = 2 * wl.n_q * d * 3 * D + 4 * len(rows) * nkv * D + 2 * len(rows) * D * d
+    return _reference_line(
+        args, world, BLOCK_METRIC, flops * len(times) / total / 1e12, total, len(times),
+        {"workload": describe(wl) + f", d_model {d}"},
+        f"per step: one full-window chunk of {wl.name}, head 0 of {wl.heads}: its q/k/v "
+        f"projection for all {wl.n_q} tokens, RoPE, append, exact fp64 attention and its "
+        f"output-projection share for {len(rows)} query rows")
 
 
 def main():
@@ -705,14 +792,17 @@ def main():
         ap.error("--warmup must be >= 3")
     from paper_2607_18171_gb300 import synth
     world, rank, local = init_dist()
-    if args.workload in synth.CONV_WORKLOADS and args.impl != "reference":
-        line = run_gpu_conv(args, synth.CONV_WORKLOADS[args.workload], world, rank, local)
+    if args.workload in synth.CONV_WORKLOADS:
+        cw = synth.CONV_WORKLOADS[args.workload]
+        line = (run_reference_conv(args, cw, world, rank) if args.impl == "reference"
+                else run_gpu_conv(args, cw, world, rank, local))
         if line is not None:
             print(json.dumps(line), flush=True)
         return
     wl = synth.WORKLOADS[args.workload]
     if args.impl == "reference":
-        line = run_reference(args, wl, world, rank)
+        line = (run_reference_block(args, wl, world, rank) if wl.block
+                else run_reference(args, wl, world, rank))
     else:
         line = run_gpu(args, wl, world, rank, local)
     if line is not None:
