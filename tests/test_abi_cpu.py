@@ -117,6 +117,15 @@ def test_calls_before_configure_are_state_errors(frt):
     L.frt_stream_destroy(None)
 
 
+def test_missing_library_fails_loudly(monkeypatch):
+    """No CPU fallback: without libfrt.so the binding raises instead of computing."""
+    from paper_2607_18171_gb300 import frt as m
+    monkeypatch.setattr(m, "_lib", None)
+    monkeypatch.setattr(m, "LIB_PATH", os.path.join(ROOT, "no-such-dir", "libfrt.so"))
+    with pytest.raises(RuntimeError, match="no CPU fallback"):
+        m.lib()
+
+
 def test_product_path_does_not_import_the_oracle():
     pkg = os.path.join(ROOT, "paper_2607_18171_gb300")
     for dirpath, _, files in os.walk(pkg):
