@@ -212,6 +212,7 @@ TINY_SHAPES = [
     (1, 8, 2, 2, 1, 2),
     (2, 8, 1, 3, 2, 3),
     (1, 12, 2, 1, 3, 1),
+    (2, 8, 1, 1, 1, 3),     # one token per chunk (the GPU's one-token edge case)
 ]
 
 
