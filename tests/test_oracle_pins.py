@@ -362,3 +362,124 @@ def test_mutant_streams_are_caught_by_bruteforce(mutant):
     qs, ks, vs, outs, _, st = run_stream(mutant, shape, 4, 7)
     bf = full_sequence_bruteforce(qs, ks, vs, shape[5], 1.0 / math.sqrt(8))
     assert max_dev(outs, bf) > 1e-6
+
+
+# ---------------------------------------------------------------------------
+# the stored-precision branch: rotated q and k rounded to bf16 (exact=False),
+# which is what every GPU parity test compares against
+# ---------------------------------------------------------------------------
+def _bf16_round_bits(x: float) -> float:
+    """Round one float64 to the nearest bfloat16 value, ties to even, by integer
+    arithmetic on its IEEE-754 bit pattern (independent of the oracle's frexp / rint
+    route). Inputs here are normal and far from the overflow edge."""
+    import struct
+    if x == 0.0:
+        return x
+    bits = struct.unpack("<Q", struct.pack("<d", x))[0]
+    sign = bits >> 63
+    exp = (bits >> 52) & 0x7FF
+    mant = (bits & ((1 << 52) - 1)) | (1 << 52)        # 53 significant bits
+    drop = 53 - 8                                       # keep 8 significant bits
+    keep, rest = mant >> drop, mant & ((1 << drop) - 1)
+    half = 1 << (drop - 1)
+    if rest > half or (rest == half and (keep & 1)):
+        keep += 1
+    value = math.ldexp(keep, exp - 1075 + drop)
+    return -value if sign else value
+
+
+def _rotate_pure_python(x, chunk, gh, gw, frames, split, theta=10000.0):
+    """3D RoPE written token by token and pair by pair with the math module."""
+    nq, nh, dim = x.shape
+    out = np.array(x, dtype=np.float64)
+    tpf = gh * gw
+    for i in range(nq):
+        f, rem = divmod(i, tpf)
+        r, col = divmod(rem, gw)
+        pos = (chunk * frames + f, r, col)
+        off = 0
+        for a in range(3):
+            width = split[a]
+            for j in range(width // 2):
+                ang = pos[a] * math.pow(theta, -2.0 * j / width)
+                c, s = math.cos(ang), math.sin(ang)
+                for h in range(nh):
+                    x0 = float(x[i, h, off + 2 * j])
+                    x1 = float(x[i, h, off + 2 * j + 1])
+                    out[i, h, off + 2 * j] = x0 * c - x1 * s
+                    out[i, h, off + 2 * j + 1] = x0 * s + x1 * c
+            off += width
+    return out
+
+
+def _bf16_pure_python(a):
+    return np.vectorize(_bf16_round_bits, otypes=[np.float64])(a)
+
+
+def test_bf16_bit_rounding_helper_matches_torch():
+    """The helper above is itself checked against torch's fp32 -> bf16 conversion on
+    fp32-representable inputs (where one rounding is all there is), ties included."""
+    x = np.concatenate([RNG.standard_normal(4000).astype(np.float32),
+                        np.array([1.0 + 2.0**-8, 1.0 + 3 * 2.0**-8, -(1.0 + 2.0**-8)],
+                                 np.float32)])
+    ref = torch.from_numpy(x).to(torch.bfloat16).to(torch.float64).numpy()
+    assert np.array_equal(_bf16_pure_python(x.astype(np.float64)), ref)
+
+
+def _stored_precision_reference(shape, n_chunks, seed):
+    """Per chunk: independently rotated, independently bf16-rounded q and k, and v."""
+    heads, dim, gh, gw, frames, window = shape
+    split = synth.default_split(dim)
+    qs, ks, vs = [], [], []
+    for c in range(n_chunks):
+        q, k, v = (synth.as_f64(t) for t in synth.random_qkv(frames * gh * gw, heads, dim, [seed, c]))
+        qs.append(_bf16_pure_python(_rotate_pure_python(q, c, gh, gw, frames, split)))
+        ks.append(_bf16_pure_python(_rotate_pure_python(k, c, gh, gw, frames, split)))
+        vs.append(v)
+    return qs, ks, vs
+
+
+def _run_stored_precision(stream_cls, shape, n_chunks, seed):
+    heads, dim, gh, gw, frames, window = shape
+    st = stream_cls(heads, dim, gh, gw, frames, window, synth.default_split(dim), exact=False)
+    outs = []
+    for c in range(n_chunks):
+        q, k, v = (synth.as_f64(t) for t in synth.random_qkv(st.n_q, heads, dim, [seed, c]))
+        outs.append(st.step(q, k, v)[0])
+    return outs, st
+
+
+@pytest.mark.parametrize("shape", TINY_SHAPES)
+def test_stored_precision_stream_matches_bruteforce_on_rounded_rotations(shape):
+    """OracleStream(exact=False) rounds the rotated q and k to bf16 before attending
+    (they are stored in bf16). Its outputs equal the pure-Python full-sequence brute
+    force fed with bf16(rotate(q)), bf16(rotate(k)) built independently."""
+    n_chunks = 4
+    qs, ks, vs = _stored_precision_reference(shape, n_chunks, 21)
+    outs, st = _run_stored_precision(O.OracleStream, shape, n_chunks, 21)
+    bf = full_sequence_bruteforce(qs, ks, vs, shape[5], st.scale)
+    assert max_dev(outs, bf) < 1e-12
+    # and the cache holds exactly the rounded rotated keys, in window order
+    k_cached, _ = st.cached_kv()
+    assert np.array_equal(k_cached, np.concatenate(ks[max(0, n_chunks - shape[5]):]))
+
+
+class _StreamLeavesKUnrounded(O.OracleStream):
+    def rope(self, q, k):   # mistake: only q is rounded
+        args = (self.chunk, self.grid_h, self.grid_w, self.frames_per_chunk, self.split, self.theta)
+        return O.bf16_round(O.rope3d(q, *args)), O.rope3d(k, *args)
+
+
+class _StreamRoundsBeforeRotating(O.OracleStream):
+    def rope(self, q, k):   # mistake: rounds the inputs, then rotates
+        args = (self.chunk, self.grid_h, self.grid_w, self.frames_per_chunk, self.split, self.theta)
+        return O.rope3d(O.bf16_round(q), *args), O.rope3d(O.bf16_round(k), *args)
+
+
+@pytest.mark.parametrize("mutant", [_StreamLeavesKUnrounded, _StreamRoundsBeforeRotating])
+def test_mutant_rounding_orders_are_caught(mutant):
+    shape = (2, 8, 1, 3, 2, 3)
+    qs, ks, vs = _stored_precision_reference(shape, 4, 21)
+    outs, st = _run_stored_precision(mutant, shape, 4, 21)
+    bf = full_sequence_bruteforce(qs, ks, vs, shape[5], st.scale)
+    assert max_dev(outs, bf) > 1e-6
