@@ -3,6 +3,10 @@ attention) on GB300, one JSON line on rank 0.
 
 A step is one frame chunk through the whole path (frt_chunk_step: RoPE-K fused into
 the append, RoPE-Q fused into the attention prologue) at steady state (full window).
+The default workload is the largest single-GPU one, stream720p (40 heads x 128, 45x80
+latent grid, 3 frames per chunk: Nq 10800, window 6 chunks: Nkv 64800). Workloads
+streamed past their window (dit14b: 20 chunks) add a per-chunk leg: every chunk of a
+fresh stream timed on its own.
 value = attention FLOPs of all ranks' steps / max-over-ranks wall time of the timed
 steps (CUDA events); ms_per_step = ms per frame chunk.
 
@@ -34,6 +38,7 @@ sys.path.insert(0, ROOT)
 METRIC = "chunk-attention TFLOP/s and ms per frame-chunk at 1 GB300; % of bf16 peak"
 UNIT = "TFLOP/s"
 POOL = 8  # distinct chunk inputs cycled through (larger than L2 for the 1.3B shape)
+CPU_HEADS = 12  # heads of the CPU-baseline sample (the whole 1.3B shape)
 
 
 def describe(wl) -> str:
@@ -245,6 +250,7 @@ def run_gpu(args, wl, world, rank, local):
     st.sync()
     e2e_ms = max_over_ranks((time.perf_counter() - w0) * 1e3, world, dev)
     e2e_value = flops * n_e2e * world / (e2e_ms * 1e-3) / 1e12
+    per_chunk = per_chunk_leg(st, wl, sid, dev, stream, local) if wl.chunks > wl.window else None
     st.close()
     if world > 1:
         torch.distributed.destroy_process_group()
@@ -281,9 +287,54 @@ def run_gpu(args, wl, world, rank, local):
                 "steps": n_e2e, "ms_per_step": round(e2e_ms / n_e2e, 4)},
         "gpu_launches": 2 * n,
     }
+    if per_chunk is not None:
+        line["per_chunk"] = per_chunk
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, seconds=args.cpu_seconds)
     return line
+
+
+PER_CHUNK_REPS = 4
+
+
+def per_chunk_leg(st, wl, sid, dev, stream, local):
+    """Every chunk of a fresh stream of ``wl.chunks`` chunks (the window grows, then
+    stays full while chunks are evicted): the attention launch of each chunk timed with
+    CUDA events, median of PER_CHUNK_REPS runs, each on a reset stream with the same
+    inputs (resident in HBM before the first run). Reported per chunk and as the mean
+    over the steady state (chunks whose window is full)."""
+    import torch
+    inputs = [tuple(t.to(dev) for t in synth_chunk(wl, sid, c)) for c in range(wl.chunks)]
+    out = st.new_out()
+    evs = timing_events(wl.chunks * PER_CHUNK_REPS, stream)
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        for r in range(PER_CHUNK_REPS):
+            st.reset()
+            for c in range(wl.chunks):
+                st.set_attention_events(*evs[r * wl.chunks + c])
+                q, k, v = inputs[c]
+                st.chunk_step(q, k, v, out)
+            st.sync()
+        torch.cuda.synchronize()
+    st.set_attention_events(None, None)
+    ms = [statistics.median(evs[r * wl.chunks + c][0].elapsed_time(evs[r * wl.chunks + c][1])
+                            for r in range(PER_CHUNK_REPS)) for c in range(wl.chunks)]
+    tf = [wl.attn_flops(c) / (m * 1e-3) / 1e12 for c, m in enumerate(ms)]
+    steady = list(range(wl.window - 1, wl.chunks))
+    steady_ms = statistics.mean(ms[c] for c in steady)
+    steady_tf = sum(wl.attn_flops(c) for c in steady) / (sum(ms[c] for c in steady) * 1e-3) / 1e12
+    return {"chunks": wl.chunks, "reps": PER_CHUNK_REPS, "statistic": "median over reps",
+            "n_kv": [wl.n_kv(c) for c in range(wl.chunks)],
+            "attention_ms": [round(m, 4) for m in ms], "tflops": [round(t, 1) for t in tf],
+            "steady_state": {"chunks": f"{steady[0]}-{steady[-1]}", "mean_ms": round(steady_ms, 4),
+                             "tflops": round(steady_tf, 1)},
+            "clocks": clk.summary()}
+
+
+def synth_chunk(wl, sid, c):
+    from paper_2607_18171_gb300 import synth
+    return synth.chunk_qkv(wl, sid, c)
 
 
 def run_gpu_multi(args, wl, world, rank, local, dev, peak_tf, peak_kind):
@@ -644,18 +695,19 @@ def cpu_baseline(wl, seconds: float = 15.0):
     TFLOP/s = attention flops of the sampled rows / step time."""
     if wl.streams > 1:
         return None
-    orc = _oracle_stream(wl, 0, wl.heads)
+    heads = min(wl.heads, CPU_HEADS)   # heads are independent: a head subset is a sample
+    orc = _oracle_stream(wl, 0, heads)
     nkv = wl.window * wl.n_q
     probe = _rows_for(wl.n_q, 64)
     dt = _oracle_step(orc, wl, 0, wl.window - 1, probe)      # window now full
     rows = _rows_for(wl.n_q, len(probe) * seconds / max(dt, 1e-3))
     dt = _oracle_step(orc, wl, 0, wl.window, rows)          # evicts chunk 0, still full
-    flops = 4 * len(rows) * nkv * wl.head_dim * wl.heads
+    flops = 4 * len(rows) * nkv * wl.head_dim * heads
     return {"value": round(flops / dt / 1e12, 6), "unit": UNIT, "cores": cpu_threads(),
             "kind": "oracle",
             "sample": f"one full-window chunk step of {wl.name}: RoPE of the chunk + append + "
                       f"exact fp64 attention for {len(rows)} of {wl.n_q} query rows x "
-                      f"{wl.heads} heads ({dt:.1f} s)"}
+                      f"{heads} of {wl.heads} heads ({dt:.1f} s)"}
 
 
 def _reference_line(args, world, metric, value, total, n, config, sample):
@@ -780,9 +832,9 @@ def run_reference_block(args, wl, world, rank):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=1000)
-    ap.add_argument("--warmup", type=int, default=20)
-    ap.add_argument("--workload", default="dit1p3b")
+    ap.add_argument("--steps", type=int, default=60)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--workload", default="stream720p")
     ap.add_argument("--impl", default="frt", choices=["frt", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)

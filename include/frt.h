@@ -245,8 +245,10 @@ frt_status frt_chunk_attention_batched(frt_stream_t* const* streams, int n,
  * lives in one static device array of this library (8 MiB of partials, 4096 merge
  * counters) that every GPU loading the library holds until exit; splits are limited
  * to what it holds, and heads * ceil(n_q / 256) > 4096 is rejected with
- * FRT_ERR_UNSUPPORTED. The first call on a device looks up the array's device
- * address; make that first call before any stream capture. All calls share the
+ * FRT_ERR_UNSUPPORTED. The first call in each CUDA context (the device's primary
+ * context, another context the caller made current, or a new primary context after
+ * cudaDeviceReset) looks up the array's device address in that context; make that
+ * first call before any stream capture. All calls share the
  * array and each clears its merge counters on the stream first: calls that overlap
  * on the GPU (other streams, other threads) race and must not be issued.
  * frt_last_error() describes an error this call returns. */

@@ -729,8 +729,9 @@ template <int D, int MAXS, bool ROPE>
 cudaError_t launch(const AttnParams<MAXS>& p, cudaStream_t st) {
     if (p.total_items <= 0) return cudaSuccess;
     auto kern = attn_kernel<D, MAXS, ROPE>;
-    static bool attr_set = false;
-    if (!attr_set) {
+    static bool attr_set[kMaxDevices] = {};   // per device: attributes are per device
+    const int dev = device_slot();
+    if (dev < 0 || !attr_set[dev]) {
         // the setmaxnreg split assumes exactly kRegsLaunch registers per thread at launch;
         // any other allocation could leave the increase waiting, so refuse to launch
         cudaFuncAttributes fa;
@@ -740,7 +741,7 @@ cudaError_t launch(const AttnParams<MAXS>& p, cudaStream_t st) {
         e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  Cfg<D>::SMEM);
         if (e != cudaSuccess) return e;
-        attr_set = true;
+        if (dev >= 0) attr_set[dev] = true;
     }
     kern<<<p.total_items, kThreads, Cfg<D>::SMEM, st>>>(p);
     return cudaGetLastError();

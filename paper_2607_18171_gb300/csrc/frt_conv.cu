@@ -468,12 +468,13 @@ template <int BN, bool PAIR>
 cudaError_t launch_conv(ConvParams p, cudaStream_t st) {
     using C = CCfg<BN, PAIR>;
     const int smem = p.a_stages * p.a_bytes + p.b_stages * p.b_stage + kSlab + 1024;
-    static int attr = 0;
-    if (smem > attr) {
+    static int attr[kMaxDevices] = {};   // per device: the largest size set so far
+    const int dev = device_slot();
+    if (dev < 0 || smem > attr[dev]) {
         cudaError_t e = cudaFuncSetAttribute(conv_kernel<BN, PAIR>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         if (e != cudaSuccess) return e;
-        attr = smem;
+        if (dev >= 0) attr[dev] = smem;
     }
     const int units = std::min(p.n_tiles, num_sms() / C::CM);
     if (!PAIR) {

@@ -404,12 +404,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
 template <int BN, bool PAIR>
 cudaError_t launch(const GemmParams& p, cudaStream_t st) {
     using C = GCfg<BN, PAIR>;
-    static bool attr_set = false;
-    if (!attr_set) {
+    static bool attr_set[kMaxDevices] = {};   // per device: attributes are per device
+    const int dev = device_slot();
+    if (dev < 0 || !attr_set[dev]) {
         cudaError_t e = cudaFuncSetAttribute(gemm_kernel<BN, PAIR>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
         if (e != cudaSuccess) return e;
-        attr_set = true;
+        if (dev >= 0) attr_set[dev] = true;
     }
     const int n_ctiles = ((p.tiles_m + C::CM - 1) / C::CM) * p.tiles_n;
     const int units = n_ctiles < num_sms() / C::CM ? n_ctiles : num_sms() / C::CM;

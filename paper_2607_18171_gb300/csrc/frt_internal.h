@@ -175,7 +175,21 @@ cudaError_t launch_attention_single(const AttnParams<1>& p, int head_dim, bool r
                                     cudaStream_t st);
 cudaError_t launch_attention_batched(const AttnParams<kMaxBatchStreams>& p, int head_dim,
                                      cudaStream_t st);
+// SM count of the calling thread's current device (cached per device).
 int num_sms();
+// One-time launch set-up (function attributes, SM counts) is per device: a function
+// attribute set with cudaFuncSetAttribute applies to the current device only. Launchers
+// keep such state in arrays indexed by this slot: the current device's ordinal, or -1
+// when it cannot be read or is beyond kMaxDevices (the set-up is then redone every call).
+constexpr int kMaxDevices = 64;
+inline int device_slot() {
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+        (void)cudaGetLastError();
+        return -1;
+    }
+    return dev;
+}
 // Set the thread-local message that frt_last_error() returns.
 void set_last_error(const char* msg);
 // Report a CUDA runtime call of the library that failed: the message is kept for

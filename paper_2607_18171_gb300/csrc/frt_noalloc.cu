@@ -11,6 +11,8 @@
 #include <cmath>
 #include <cstring>
 #include <mutex>
+#include <utility>
+#include <vector>
 
 #include "../../include/frt.h"
 #include "frt_internal.h"
@@ -28,14 +30,49 @@ constexpr size_t kScratchBytes = kPartBytes + kMlBytes + size_t(kMaxGroups) * si
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kScratchBytes];
 
-constexpr int kMaxDevices = 64;
+// Device address of g_noalloc_scratch per CUDA context. A __device__ symbol's address
+// belongs to the context that loaded the module, so the cache is keyed by the context's
+// unique ID (cuCtxGetId: never reused within a process), not by the device ordinal: a
+// non-primary context, or the new primary context after a cudaDeviceReset, looks the
+// address up again instead of using a stale one.
 std::mutex g_mu;
-void* g_scratch_dev[kMaxDevices] = {};   // device address of g_noalloc_scratch per device
+std::vector<std::pair<unsigned long long, void*>> g_scratch_by_ctx;
+
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+template <typename Fn>
+Fn driver_fn(const char* name) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion(name, &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+        return reinterpret_cast<Fn>(p);
+    return nullptr;
+}
+
+// Unique ID of the calling thread's current context; 0 if none is current or the driver
+// does not offer the query.
+unsigned long long current_ctx_id() {
+    static CtxGetCurrentFn get_cur = nullptr;
+    static CtxGetIdFn get_id = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        get_cur = driver_fn<CtxGetCurrentFn>("cuCtxGetCurrent");
+        get_id = driver_fn<CtxGetIdFn>("cuCtxGetId");
+    });
+    CUcontext ctx = nullptr;
+    unsigned long long id = 0;
+    if (!get_cur || !get_id || get_cur(&ctx) != CUDA_SUCCESS || ctx == nullptr ||
+        get_id(ctx, &id) != CUDA_SUCCESS)
+        return 0;
+    return id;
+}
 
 EncodeTiledFn encode_fn() {
     static EncodeTiledFn fn = nullptr;
@@ -128,23 +165,26 @@ extern "C" frt_status frt_chunk_attention_noalloc(const void* q, const void* k, 
                     "heads * ceil(n_q / 256) exceeds the static maximum of 4096 query groups; "
                     "use frt_chunk_attention for larger chunks");
 
-    // one-time set-up per device: the array's device address (host code may not use
-    // the symbol itself as a device pointer)
+    // one-time set-up per context: the array's device address (host code may not use
+    // the symbol itself as a device pointer). The look-up also makes the device's primary
+    // context current when the calling thread has none yet.
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess || dev < 0 || dev >= kMaxDevices)
-        return cuda_failed("no usable current device");
+    if (e != cudaSuccess) return cuda_failed("no usable current device");
     void* base = nullptr;
     {
         std::lock_guard<std::mutex> lock(g_mu);
-        if (!g_scratch_dev[dev]) {
-            void* ptr = nullptr;
-            e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
-            if (e != cudaSuccess || !ptr)
+        unsigned long long ctx = current_ctx_id();
+        for (const auto& entry : g_scratch_by_ctx)
+            if (ctx != 0 && entry.first == ctx) base = entry.second;
+        if (!base) {
+            e = cudaGetSymbolAddress(&base, g_noalloc_scratch);
+            if (e != cudaSuccess || !base)
                 return cuda_failed("cudaGetSymbolAddress of the static scratch failed");
-            g_scratch_dev[dev] = ptr;
+            if (ctx == 0) ctx = current_ctx_id();
+            if (ctx == 0) return fail(FRT_ERR_CUDA, "no current CUDA context after set-up");
+            g_scratch_by_ctx.emplace_back(ctx, base);
         }
-        base = g_scratch_dev[dev];
     }
     uint8_t* b = static_cast<uint8_t*>(base);
     float* part_o = reinterpret_cast<float*>(b);

@@ -169,13 +169,14 @@ cudaError_t launch_staged(StagedParams& sp, cudaStream_t st) {
     if (sp.stages < 2) return cudaErrorInvalidValue;   // rows too large (create() prevents it)
     sp.wait_limit_ns = 2000000000ull;
     const int smem = sp.stages * stage_bytes;
-    static bool attr = false;
-    if (!attr) {
+    static bool attr[kMaxDevices] = {};   // per device: attributes are per device
+    const int dev = device_slot();
+    if (dev < 0 || !attr[dev]) {
         cudaError_t e = cudaFuncSetAttribute(staged_rows_kernel,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              kSmemBudget);
         if (e != cudaSuccess) return e;
-        attr = true;
+        if (dev >= 0) attr[dev] = true;
     }
     const int n_blocks = (sp.n_tok + sp.tok_per_block - 1) / sp.tok_per_block;
     const int grid = std::min(n_blocks, num_sms());
@@ -185,16 +186,17 @@ cudaError_t launch_staged(StagedParams& sp, cudaStream_t st) {
 }  // namespace
 
 int num_sms() {
-    static int n = 0;
-    if (n == 0) {
-        int dev = 0, v = 0;
-        if (cudaGetDevice(&dev) == cudaSuccess &&
-            cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess)
-            n = v;
-        else
-            n = 148;
+    static int n[kMaxDevices] = {};   // per device: devices may differ
+    const int dev = device_slot();
+    if (dev >= 0 && n[dev] > 0) return n[dev];
+    int v = 0;
+    if (dev < 0 || cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        v <= 0) {
+        (void)cudaGetLastError();
+        return 148;   // no readable device (host-only planning calls)
     }
-    return n;
+    n[dev] = v;
+    return v;
 }
 
 cudaError_t launch_kv_append(const AppendParams& p, cudaStream_t st) {
