@@ -62,7 +62,10 @@ typedef struct frt_config {
     void* cuda_stream;             /* cudaStream_t all work is enqueued on; NULL = legacy stream */
 } frt_config;
 
-/* Create a stream handle.
+/* Create a stream handle: one (video stream, denoising step) and its persistent KV
+ * cache, the cross-batch state that batch j inherits from batch j-1 (paper section 2
+ * "Problem Formulation", the lambda = 1 edge; Appendix A.1.2 "Pipeline graph"); chunks
+ * of frames_per_chunk frames are the batches (Appendix A.1.1 "Initial assumptions").
  *   heads >= 1; head_dim in {64, 128}; heads * head_dim <= 12800; tokens_per_frame >= 1;
  *   frames_per_chunk >= 1; window_chunks >= 1 (the window counts the current chunk).
  * Nq = frames_per_chunk * tokens_per_frame must be <= 2^20 and
@@ -83,7 +86,10 @@ frt_status frt_config_default(const frt_stream_t* s, frt_config* cfg);
  * calls return FRT_ERR_STATE until a configure succeeds. */
 frt_status frt_stream_configure(frt_stream_t* s, const frt_config* cfg);
 
-/* Operation 1: rotate q and k (bf16 [Nq, heads, head_dim]) in place at the
+/* Operation 1 (the paper does not define the position encoding: it deploys video DiTs,
+ * sections 4.3.3-4.3.4, whose attention runs on rotated q and k; the segment split and
+ * pairing are this library's convention, fixed by frt_config):
+ * rotate q and k (bf16 [Nq, heads, head_dim]) in place at the
  * positions of chunk c = frt_stream_chunk_counter(s): token i sits at
  * (t = c * frames_per_chunk + i / tokens_per_frame, row, column); in segment
  * a of width d_a, pair (2j, 2j+1) turns by pos_a * theta^(-2j/d_a).
@@ -91,7 +97,10 @@ frt_status frt_stream_configure(frt_stream_t* s, const frt_config* cfg);
  * attention); otherwise FRT_ERR_STATE. */
 frt_status frt_rope3d_qk(frt_stream_t* s, void* q, void* k);
 
-/* Operation 2: copy the rotated k and v of chunk c into ring slot c mod W
+/* Operation 2, the write side of the KV-cache state edge (section 2 "Problem
+ * Formulation"; section 3.2 "IR design": a node's persistent-state writes; Appendix
+ * A.1.2: the cache batch j+1 inherits from batch j): copy the rotated k and v of chunk
+ * c into ring slot c mod W
  * (cache rows [slot*Nq, (slot+1)*Nq)), overwriting evicted chunk c - W, then
  * advance the counter. *slot_out = c mod W, *evicted_out = c - W or -1 (either
  * pointer may be NULL). Indices are computed on the host (exact). Must follow
@@ -99,7 +108,9 @@ frt_status frt_rope3d_qk(frt_stream_t* s, void* q, void* k);
 frt_status frt_kv_append_evict(frt_stream_t* s, const void* k, const void* v,
                                int* slot_out, long long* evicted_out);
 
-/* Operation 3: out[i, h, :] = sum_j softmax_j(sm_scale * <q[i,h], K[j,h]>) V[j,h,:]
+/* Operation 3, the read side of that state edge inside the DiT, the stage that sets the
+ * pipelines' frame-rate ceiling (Appendix B.1 "What drives the tradeoff"):
+ * out[i, h, :] = sum_j softmax_j(sm_scale * <q[i,h], K[j,h]>) V[j,h,:]
  * over every valid cached row j (n_c * Nq rows, n_c = min(c + 1, W) for the
  * chunk c just appended): bidirectional inside the chunk, all earlier chunks
  * of the window. bf16 operands, fp32 accumulation, P rounded to bf16 for the
@@ -110,7 +121,8 @@ frt_status frt_kv_append_evict(frt_stream_t* s, const void* k, const void* v,
 frt_status frt_chunk_attention(const void* q, const void* k, const void* v,
                                void* out, frt_stream_t* s);
 
-/* Operations 1-3 fused for one chunk: q, k, v are the raw (unrotated) inputs
+/* Operations 1-3 fused for one chunk (one batch's pass over the state edge of section 2
+ * and Appendix A.1.2): q, k, v are the raw (unrotated) inputs
  * and are not modified; RoPE-K runs inside the append (rotated K goes to the
  * cache only) and RoPE-Q inside the attention kernel's prologue. Same result
  * as the three separate calls. Allowed at the start of a chunk. */
@@ -216,7 +228,9 @@ frt_status frt_conv_sync(frt_conv_t* c);
 frt_status frt_conv_reset(frt_conv_t* c);
 void frt_conv_destroy(frt_conv_t* c);
 
-/* Operation 3 for n independent streams in one launch (ragged KV lengths):
+/* Operation 3 for n independent streams in one launch (ragged KV lengths; streams hold
+ * disjoint persistent state, so they carry no cross-stream edge: section 3.2 "IR
+ * design", node-level state annotation):
  * each streams[i] must have just appended (as for frt_chunk_attention); q[i]
  * and out[i] are that stream's rotated queries and output. All streams must
  * share heads, head_dim, sm_scale and out dtype; work is ordered longest KV
@@ -279,11 +293,13 @@ frt_status frt_steps_tick(frt_steps_t* g, unsigned int active_mask, void* const*
                           void* const* k, const void* const* v, void* const* out);
 void frt_steps_destroy(frt_steps_t* g);
 
-/* Wait for the stream's work and return its device status (FRT_OK or the
+/* Wait for the stream's work and return its device status (no counterpart in the
+ * paper; the library's error channel) (FRT_OK or the
  * first device error, e.g. FRT_ERR_TIMEOUT). */
 frt_status frt_stream_sync(frt_stream_t* s);
 
-/* Clear the cache contents, chunk counter, ordering state, split-KV merge
+/* Start the stream over, as a new video would (the state edge of section 2 has no
+ * predecessor for batch 0): clear the cache contents, chunk counter, ordering state, split-KV merge
  * counters and device status (the way back after FRT_ERR_TIMEOUT). */
 frt_status frt_stream_reset(frt_stream_t* s);
 

@@ -9,11 +9,14 @@
 // setmaxnreg: warpgroup 0 drops to kRegsCtl, the two softmax warpgroups rise to kRegsSm.
 //   warp 0      TMA producer: Q tiles once, then K/V tiles (K0, V0, K1, V1, ...) through
 //               a STAGES-deep shared-memory ring.
-//   warp 1      TMEM allocator + single-thread tcgen05.mma issuer:
+//   warp 1      TMEM allocator + tcgen05.mma issuer (converged warp, lane 0 issues):
 //                 S_g  = Q_g K_j^T  A, B from shared memory (K-major, 128-byte swizzle)
 //                 O_g += P_g V_j    A = P from TMEM, B = V from shared memory (MN-major)
 //               issued as PV_0(j), S_0(j+1), PV_1(j), S_1(j+1): the tiles alternate
-//   warps 2-3   idle
+//   warp 2      observer: waits on the K/V and P barriers the issuer needs next and hands
+//               off to it through a named barrier (the issuer touches no mbarrier in the
+//               KV loop)
+//   warp 3      idle
 //   warps 4-7   softmax group 0 (query tile 0), one thread per query row
 //   warps 8-11  softmax group 1 (query tile 1)
 // TMEM (512 columns): S_0 [0,128), S_1 [128,256), O_0 [256,256+D), O_1 [256+D,256+2D).
@@ -47,6 +50,9 @@ constexpr int kBM = 128;   // query rows per tile
 constexpr int kBN = 128;   // KV rows per tile
 constexpr float kOverflowGuard = 1.152921504606846976e18f;   // 2^60
 constexpr int kTimeoutCode = 6;  // FRT_ERR_TIMEOUT
+// Named barrier of the issuer / observer hand-off (warps 1 and 2). Ids 1-3 serve the
+// softmax groups' epilogues, id 0 is __syncthreads.
+constexpr int kBarHandoff = 4;
 
 template <int D>
 struct Cfg {
@@ -214,132 +220,115 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             mbar_wait_drain(qbar, 0, lim);
         }
       } else if (warp == 1) {
-        // ============ MMA issuer: one thread, tiles alternate on the tensor pipe ============
-        if (lane == 0) {
-            bool ok = true;
-            for (int g = 0; g < ng && ok; ++g)
-                if (!mbar_wait(smem_u32(&bars->q_ready[g]), 0, lim, abort)) {
-                    report(p.status, abort, 1, -1 - g);
-                    ok = false;
-                }
+        // ===== MMA issuer: a converged warp whose lane 0 issues; tiles alternate on the pipe =====
+        // The warp never touches an mbarrier inside the KV loop: the observer warp (warp 2)
+        // waits for every load and P barrier the next MMAs need and meets this warp at the
+        // hand-off named barrier. A shared-memory access by the issuing thread behind queued
+        // MMAs costs it more than an MMA's shadow (the MMAs' operand reads keep shared memory
+        // busy); a named barrier is a hardware barrier and touches no shared memory.
+        const uint32_t lead = (lane == 0) ? 1u : 0u;
+        bool ok = true;
+        for (int g = 0; g < ng && ok; ++g)
+            if (!mbar_wait(smem_u32(&bars->q_ready[g]), 0, lim, abort)) {
+                if (lane == 0) report(p.status, abort, 1, -1 - g);
+                ok = false;
+            }
+        ok = __all_sync(0xffffffffu, ok);
+        // after an error no MMA is issued, but every hand-off still takes place: the
+        // observer and this warp always pass the same number of barriers
+        const uint32_t iss = ok ? lead : 0u;
+        tc_fence_after();
+        // tcgen05.mma issue blocks until the tensor pipe has (nearly) drained the previous
+        // MMA, so every instruction between MMAs is tensor idle time: the descriptors are
+        // precomputed and advanced by constant adds (a descriptor is linear in its 16-byte
+        // start address; addresses stay below 256 KB, no carry).
+        const uint64_t dq0 = sdesc_sw128(sQ, 16, 1024);
+        const uint64_t dk0 = sdesc_sw128(sKV, 16, 1024);
+        const uint64_t dv0 = sdesc_sw128(sKV, kBN * 128, 1024);
+        // one hand-off: the observer has seen the next awaited barrier complete (or gave up
+        // and raised the abort flag; the MMAs then compute on stale operands, which the
+        // error status marks as void)
+        auto handoff = [&]() {
+            named_bar_sync(kBarHandoff, 64);
             tc_fence_after();
-            // tcgen05.mma issue blocks until the tensor pipe has (nearly) drained the
-            // previous MMA, so every instruction between MMAs is tensor idle time: the
-            // descriptors are precomputed and advanced by constant adds (a descriptor is
-            // linear in its 16-byte start address; addresses stay below 256 KB, no carry).
-            const uint64_t dq0 = sdesc_sw128(sQ, 16, 1024);
-            const uint64_t dk0 = sdesc_sw128(sKV, 16, 1024);
-            const uint64_t dv0 = sdesc_sw128(sKV, kBN * 128, 1024);
-            // K_j and V_j share a barrier, kv_full[j % 4]: waiting for K_j (load 2j)
-            // covers V_j, so the wait for load 2j+1 is a no-op. Pair j+4 is loaded only
-            // after step j-1's slot release, which this thread commits after it waited
-            // for pair j, so the parity of kv_full[j % 4] is never ambiguous.
-            auto wait_load = [&](int Lw) -> bool {
-                if (Lw & 1) return true;
-                const uint32_t fb = smem_u32(&bars->kv_full[(Lw >> 1) & 3]);
-                const uint32_t par = ((Lw >> 1) >> 2) & 1;
-                if (!mbar_test_wait(fb, par) && !mbar_wait(fb, par, lim, abort)) {
-                    report(p.status, abort, 1, Lw);
-                    return false;
-                }
-                tc_fence_after();
-                return true;
-            };
-            // MMA groups: S_g = Q_g K^T (8 MMAs over D) and O_g += P_g V (8 MMAs over the
-            // KV tile). `mid(k)` runs after MMA k of a group, while the tensor pipe still
-            // works on it: after issuing an MMA the thread has about one MMA (64 cycles) of
-            // slack, so bookkeeping is spread one operation per gap to stay hidden.
-            auto issue_s = [&](int g, int stage, auto&& mid) {
-                const uint64_t dq = dq0 + uint64_t((g * C::Q_TILE) >> 4);
-                const uint64_t dk = dk0 + uint64_t((stage * C::KV_TILE) >> 4);
-                const uint32_t d = tmem + g * kBN;
+        };
+        // MMA groups: S_g = Q_g K^T (8 MMAs over D) and O_g += P_g V (8 MMAs over the KV
+        // tile). `mid(k)` runs after MMA k of a group, in the shadow of the running MMA.
+        auto issue_s = [&](int g, int stage, auto&& mid) {
+            const uint64_t dq = dq0 + uint64_t((g * C::Q_TILE) >> 4);
+            const uint64_t dk = dk0 + uint64_t((stage * C::KV_TILE) >> 4);
+            const uint32_t d = tmem + g * kBN;
 #pragma unroll
-                for (int k = 0; k < D / 16; ++k) {
-                    const uint64_t off = uint64_t((k >> 2) * ((kBM * 128) >> 4) + (k & 3) * 2);
-                    umma_ss(d, dq + off, dk + off, C::IDESC_S, k > 0 ? 1u : 0u);
-                    mid(k);
-                }
-                umma_commit(smem_u32(&bars->s_full[g]));
-            };
-            auto issue_o = [&](int g, int stage, bool acc, auto&& mid) {
-                const uint64_t dv = dv0 + uint64_t((stage * C::KV_TILE) >> 4);
-                const uint32_t d = tmem + 256 + g * D;
-                const uint32_t pa = tmem + g * kBN;   // P_g: bf16 pairs in S_g's columns
+            for (int k = 0; k < D / 16; ++k) {
+                const uint64_t off = uint64_t((k >> 2) * ((kBM * 128) >> 4) + (k & 3) * 2);
+                umma_ss_if(iss, d, dq + off, dk + off, C::IDESC_S, k > 0 ? 1u : 0u);
+                mid(k);
+            }
+            umma_commit_if(iss, smem_u32(&bars->s_full[g]));
+        };
+        auto issue_o = [&](int g, int stage, bool acc, auto&& mid) {
+            const uint64_t dv = dv0 + uint64_t((stage * C::KV_TILE) >> 4);
+            const uint32_t d = tmem + 256 + g * D;
+            const uint32_t pa = tmem + g * kBN;   // P_g: bf16 pairs in S_g's columns
 #pragma unroll
-                for (int k = 0; k < kBN / 16; ++k) {
-                    umma_ts(d, pa + k * 8, dv + uint64_t(k * ((16 * 128) >> 4)), C::IDESC_O,
-                            (acc || k > 0) ? 1u : 0u);
-                    mid(k);
-                }
-            };
-            auto wait_p = [&](int g, int j) -> bool {
-                if (!mbar_wait(smem_u32(&bars->p_full[g]), j & 1, lim, abort)) {
-                    report(p.status, abort, 1, 2000 + j);
-                    return false;
-                }
-                tc_fence_after();
-                return true;
-            };
-            auto nop = [](int) {};
-            // load order of the producer: K0, V0, K1, V1, ... -> load 2j is K_j, 2j+1 is V_j
-            if (ok && (ok = wait_load(0))) {
-                issue_s(0, 0, nop);
-                if (ng == 2) issue_s(1, 0, [&](int k) { if (k == 0) ok = wait_load(1); });
-                else ok = wait_load(1);
-                umma_commit(smem_u32(&bars->k0_done));
+            for (int k = 0; k < kBN / 16; ++k) {
+                umma_ts_if(iss, d, pa + k * 8, dv + uint64_t(k * ((16 * 128) >> 4)), C::IDESC_O,
+                           (acc || k > 0) ? 1u : 0u);
+                mid(k);
             }
-            int sv = 1 % C::STAGES, sk = 2 % C::STAGES;   // ring slots of V_j and K_{j+1}
-            // An MMA issue returns only once the previous MMA has drained, so a blocking
-            // wait at a group boundary idles the tensor pipe. P_g of the next PV group is
-            // therefore probed (non-blocking) from the shadow of the last MMA of the group
-            // before it; when the probe has seen it complete, only the fence remains at
-            // the boundary. One probe, not several: a shared-memory access by this thread
-            // behind queued MMAs costs it ~140 cycles, more than an MMA's shadow.
-            auto take_p = [&](int g, int j, bool seen) -> bool {
-                if (seen) {
-                    tc_fence_after();
-                    return true;
-                }
-                return wait_p(g, j);
-            };
-            auto probe_p = [&](int g, int j) -> bool {
-                return mbar_test_wait(smem_u32(&bars->p_full[g]), j & 1);
-            };
-            bool p0_seen = false, p1_seen = false;
-            for (int j = 0; j < n_tiles && ok; ++j) {
-                const bool more = (j + 1) < n_tiles;
-                // V_j has been waited for; K_{j+1} is waited for inside PV_0(j);
-                // V_{j+1} inside the last group of this step.
-                if (!(ok = take_p(0, j, p0_seen))) break;
-                p0_seen = false;
-                // the release of step j-1 rides in the shadow of PV_0(j)'s second MMA
-                // instead of idling the tensor pipe at the end of step j-1
-                issue_o(0, sv, j > 0, [&](int k) {
-                    if (k == 0 && more) ok = wait_load(2 * j + 2);
-                    if (k == 1 && j > 0) umma_commit(smem_u32(&bars->step_done[(j - 1) & 3]));
-                });
-                if (!ok) break;
-                if (ng == 2) {
-                    if (more) issue_s(0, sk, [&](int k) { if (k == D / 16 - 1) p1_seen = probe_p(1, j); });
-                    else umma_commit(smem_u32(&bars->o_done[0]));
-                    if (!(ok = take_p(1, j, p1_seen))) break;
-                    p1_seen = false;
-                    issue_o(1, sv, j > 0, nop);
-                    if (more) issue_s(1, sk, [&](int k) {
-                        if (k == 0) ok = wait_load(2 * j + 3);
-                        if (k == D / 16 - 1) p0_seen = probe_p(0, j + 1);
-                    });
-                    else umma_commit(smem_u32(&bars->o_done[1]));
-                } else {
-                    if (more) issue_s(0, sk, [&](int k) { if (k == 0) ok = wait_load(2 * j + 3); });
-                    else umma_commit(smem_u32(&bars->o_done[0]));
-                }
-                sv = (sv + 2 >= C::STAGES) ? sv + 2 - C::STAGES : sv + 2;
-                sk = (sk + 2 >= C::STAGES) ? sk + 2 - C::STAGES : sk + 2;
+        };
+        auto nop = [](int) {};
+        // Hand-off sequence (the observer follows the same one): K_0/V_0; then per KV step
+        // j: P_0(j), K_{j+1}/V_{j+1} (if any), P_1(j) (two tiles).
+        handoff();
+        issue_s(0, 0, nop);
+        if (ng == 2) issue_s(1, 0, nop);
+        umma_commit_if(iss, smem_u32(&bars->k0_done));
+        int sv = 1 % C::STAGES, sk = 2 % C::STAGES;   // ring slots of V_j and K_{j+1}
+        for (int j = 0; j < n_tiles; ++j) {
+            const bool more = (j + 1) < n_tiles;
+            handoff();                                  // P_0(j)
+            // the release of step j-1 rides in the shadow of PV_0(j)'s second MMA
+            issue_o(0, sv, j > 0, [&](int k) {
+                if (k == 0 && more) handoff();          // K_{j+1}, V_{j+1}
+                if (k == 1 && j > 0) umma_commit_if(iss, smem_u32(&bars->step_done[(j - 1) & 3]));
+            });
+            if (more) issue_s(0, sk, nop);
+            else umma_commit_if(iss, smem_u32(&bars->o_done[0]));
+            if (ng == 2) {
+                handoff();                              // P_1(j)
+                issue_o(1, sv, j > 0, nop);
+                if (more) issue_s(1, sk, nop);
+                else umma_commit_if(iss, smem_u32(&bars->o_done[1]));
             }
-            // drain: all issued MMAs complete before TMEM is released
-            umma_commit(smem_u32(&bars->drain[0]));
-            mbar_wait_drain(smem_u32(&bars->drain[0]), 0, lim);
+            sv = (sv + 2 >= C::STAGES) ? sv + 2 - C::STAGES : sv + 2;
+            sk = (sk + 2 >= C::STAGES) ? sk + 2 - C::STAGES : sk + 2;
+        }
+        // drain: all issued MMAs complete before TMEM is released
+        umma_commit_if(lead, smem_u32(&bars->drain[0]));
+        mbar_wait_drain(smem_u32(&bars->drain[0]), 0, lim);
+      } else if (warp == 2) {
+        // ===== observer: waits for what the issuer's next MMAs need, then hands off =====
+        // Every wait is bounded; after one gives up (or another role raised the abort flag)
+        // the remaining hand-offs pass without waiting, so both warps pass the same number
+        // of barriers and the issuer finishes its (void) loop.
+        bool ok = true;
+        auto observe = [&](uint32_t bar, uint32_t parity, int where) {
+            if (ok) {
+                ok = __all_sync(0xffffffffu, mbar_wait(bar, parity, lim, abort));
+                if (!ok && lane == 0) report(p.status, abort, 4, where);
+            }
+            named_bar_sync(kBarHandoff, 64);
+        };
+        // K_j and V_j (loads 2j, 2j+1) complete together on kv_full[j % 4]. Pair j+4 is
+        // loaded only after step j-1's slot release, which the issuer commits after this
+        // warp saw pair j, so the parity of kv_full[j % 4] is never ambiguous.
+        auto kv_bar = [&](int jj) { return smem_u32(&bars->kv_full[jj & 3]); };
+        observe(kv_bar(0), 0, 0);
+        for (int j = 0; j < n_tiles; ++j) {
+            observe(smem_u32(&bars->p_full[0]), j & 1, 2000 + j);
+            if (j + 1 < n_tiles) observe(kv_bar(j + 1), ((j + 1) >> 2) & 1, 2 * (j + 1));
+            if (ng == 2) observe(smem_u32(&bars->p_full[1]), j & 1, 3000 + j);
         }
       }
     } else {

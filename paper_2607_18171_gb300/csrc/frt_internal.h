@@ -17,7 +17,7 @@ constexpr int kMaxSplit = 4;
 struct DeviceStatus {
     int code;      // 0 = ok, else an frt_status value
     int block;     // blockIdx.x of the CTA that reported it
-    int role;      // 0 producer, 1 mma, 2+ softmax group
+    int role;      // 0 producer, 1 mma issuer, 2-3 softmax groups, 4 observer (attention)
     int where;     // loop iteration or barrier id
 };
 
