@@ -47,7 +47,9 @@ typedef enum frt_status {
     FRT_ERR_OOM = 3,          /* device or pinned allocation failed */
     FRT_ERR_CUDA = 4,         /* a CUDA runtime/driver call failed */
     FRT_ERR_UNSUPPORTED = 5,  /* head_dim or shape the kernels do not handle */
-    FRT_ERR_TIMEOUT = 6       /* a device-side bounded wait gave up */
+    FRT_ERR_TIMEOUT = 6,      /* a device-side bounded wait gave up */
+    FRT_ERR_BOUNDS = 7        /* a guard word around the KV cache was overwritten, or (debug
+                                 build) a kernel's bounds check refused an access */
 } frt_status;
 
 typedef enum frt_out_dtype { FRT_OUT_F32 = 0, FRT_OUT_BF16 = 1 } frt_out_dtype;
@@ -184,6 +186,17 @@ frt_status frt_gemm_bf16(const void* a, const void* b, void* c, int M, int N,
  * current device's SM count (148 assumed when no device is visible). */
 frt_status frt_gemm_plan(int M, int N, int qkv, int d, int* bn, int* ctas);
 
+/* Work split of one chunk-attention launch (for reports and tests; no counterpart in
+ * the paper). A launch runs one CTA per work item; a query group is (stream, head, 256
+ * query rows). For n streams in launch order with n_q[i] queries and n_kv[i] valid
+ * keys, all with `heads` heads, on `sms` SMs (<= 0: the current device's SM count, 148
+ * when none is visible): query groups [0, *n_full) run whole and each later group's KV
+ * range is cut into *n_split parts whose partials are merged (the plan whose simulated
+ * schedule of the launch ends first). FRT_ERR_INVALID_ARG on NULL pointers or sizes
+ * < 1. Host-only: it launches nothing. */
+frt_status frt_attention_plan(int n, const int* n_q, const long long* n_kv, int heads, int sms,
+                              int* n_full, int* n_split);
+
 /* ---- Streaming causal 3D convolution (the VAE-decoder stage) --------------------
  * The paper's video pipelines end in a streaming VAE decoder (Appendix A.3, the
  * DiT -> VAE template: the decoder carries state from one batch to the next, the
@@ -305,6 +318,33 @@ frt_status frt_stream_reset(frt_stream_t* s);
 
 /* Release everything the handle owns (waits for its work first). NULL is a no-op. */
 void frt_stream_destroy(frt_stream_t* s);
+
+/* Snapshot of the stream's persistent state (the paper's cross-batch state edge, section
+ * 2; moving it between resources is the kappa cost of Appendix A.1.2): enqueue copies of
+ * the whole ring (K and V, rows = window_chunks * Nq each, [rows, heads, head_dim] bf16)
+ * into k_dst / v_dst (device or pinned host memory, caller-owned) on the stream's CUDA
+ * stream, and report the chunk counter. The copies are complete when frt_stream_sync
+ * returns. Not allowed between frt_rope3d_qk and the append (FRT_ERR_STATE). */
+frt_status frt_stream_save(frt_stream_t* s, void* k_dst, void* v_dst, long long* counter);
+
+/* Load a snapshot taken by frt_stream_save (from this stream or another of the same
+ * shape) and continue from it: the ring is overwritten from k_src / v_src (enqueued on
+ * the stream), the counter set, and the next call must start a chunk. The chunks that
+ * follow produce the outputs the saved stream would have produced, bit for bit. */
+frt_status frt_stream_restore(frt_stream_t* s, const void* k_src, const void* v_src,
+                              long long counter);
+
+/* Race and overrun detection (no counterpart in the paper). Every ring buffer sits
+ * between guard words written at configure; this call waits for the stream's work and
+ * compares them: FRT_ERR_BOUNDS (naming the guard) if a kernel wrote past either end of
+ * the K or V ring, else FRT_OK. The FRT_DEBUG build of the library also runs it inside
+ * every frt_stream_sync, and its kernels check every derived index (work items, ring
+ * rows, split-KV rows) against the launch's extents: an access outside is skipped and
+ * FRT_ERR_BOUNDS recorded in the stream's status (no trap). */
+frt_status frt_stream_check_guards(frt_stream_t* s);
+
+/* 1 if this library was built with FRT_DEBUG (bounds-checking kernels), else 0. */
+int frt_debug_build(void);
 
 /* Read-only view of the stream's ring buffer for inspection and snapshots: device
  * pointers of the K and V caches ([rows, heads, head_dim] bf16, rows = W * Nq; chunk c

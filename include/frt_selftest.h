@@ -44,6 +44,17 @@ int frt_selftest_gemm_force_bn(int bn);
  * block, which frt_stream_sync then returns. s must be configured. */
 frt_status frt_selftest_wait_timeout(frt_stream_t* s, long long limit_ns, void* cuda_stream);
 
+/* Debug build only (FRT_DEBUG): the next append of any stream aims its stores one ring
+ * slot past the end of the cache. The kernel's bounds check must refuse them and record
+ * FRT_ERR_BOUNDS; the debug build keeps one chunk of slack after the rear guard, so the
+ * stores would still land in the library's own memory if the check missed them (and the
+ * guard check would report it). FRT_ERR_UNSUPPORTED in a release build. */
+frt_status frt_selftest_append_past_ring(void);
+
+/* Overwrite one byte of a guard word of s (which: 0 K front, 1 V front, 2 K rear, 3 V
+ * rear) from the host, to check that frt_stream_check_guards reports it. */
+frt_status frt_selftest_poke_guard(frt_stream_t* s, int which);
+
 #ifdef __cplusplus
 }
 #endif

@@ -17,6 +17,11 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libfrt.so")
+# the FRT_DEBUG variant: kernels bounds-check every derived index and record
+# FRT_ERR_BOUNDS instead of touching memory outside its buffer; every stream sync also
+# compares the guard words around the KV cache
+DEBUG_BUILD = os.path.join(PKG, "_build_debug")
+DEBUG_LIB = os.path.join(PKG, "libfrt_debug.so")
 ARCH_FLAGS = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
           "-I", os.path.join(ROOT, "include"), "--expt-relaxed-constexpr"]
@@ -41,23 +46,28 @@ def _inputs() -> list[str]:
     return files
 
 
-def _stamp() -> str:
-    return f"{platform.machine()}|{' '.join(ARCH_FLAGS + CFLAGS)}"
+def _stamp(debug: bool = False) -> str:
+    return f"{platform.machine()}|{' '.join(ARCH_FLAGS + CFLAGS)}|{'debug' if debug else ''}"
 
 
-def up_to_date() -> bool:
-    stamp = os.path.join(BUILD, "stamp")
-    if not (os.path.exists(LIB) and os.path.exists(stamp)):
+def up_to_date(debug: bool = False) -> bool:
+    build_dir, lib = (DEBUG_BUILD, DEBUG_LIB) if debug else (BUILD, LIB)
+    stamp = os.path.join(build_dir, "stamp")
+    if not (os.path.exists(lib) and os.path.exists(stamp)):
         return False
-    if open(stamp).read() != _stamp():
+    if open(stamp).read() != _stamp(debug):
         return False
-    t = os.path.getmtime(LIB)
+    t = os.path.getmtime(lib)
     return all(os.path.getmtime(f) <= t for f in _inputs())
 
 
-def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
-    """Compile and link libfrt.so; returns its path. Raises on a compiler error."""
-    if not force and not extra_flags and up_to_date():
+def build(force: bool = False, verbose: bool = False, extra_flags=(), debug: bool = False) -> str:
+    """Compile and link libfrt.so (libfrt_debug.so with debug=True, compiled with
+    -DFRT_DEBUG); returns its path. Raises on a compiler error."""
+    BUILD, LIB = (DEBUG_BUILD, DEBUG_LIB) if debug else (globals()["BUILD"], globals()["LIB"])
+    if debug:
+        extra_flags = ("-DFRT_DEBUG", *extra_flags)
+    if not force and (debug or not extra_flags) and up_to_date(debug):
         return LIB
     os.makedirs(BUILD, exist_ok=True)
     cc = nvcc()
@@ -81,11 +91,12 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
         raise RuntimeError(f"link failed:\n{r.stderr}")
     os.replace(tmp, LIB)
     with open(os.path.join(BUILD, "stamp"), "w") as f:
-        f.write(_stamp())
+        f.write(_stamp(debug))
     return LIB
 
 
 if __name__ == "__main__":
     import sys
     print(build(force="--force" in sys.argv, verbose=True,
-                extra_flags=("-Xptxas", "-v") if "--ptxas" in sys.argv else ()))
+                extra_flags=("-Xptxas", "-v") if "--ptxas" in sys.argv else (),
+                debug="--debug" in sys.argv))

@@ -4,7 +4,8 @@
 // (the whole window is visible to every query of the chunk: bidirectional within the
 // chunk, all earlier chunks of the window), bf16 operands, fp32 accumulation.
 //
-// One CTA = one work item = (stream, head, 256 query rows as two 128-row tiles).
+// One CTA = one work item = (stream, head, 256 query rows as two 128-row tiles, a range of
+// the KV tiles: all of them, or one of n_split parts for the groups of the last waves).
 // Three warpgroups (384 threads, one CTA per SM); registers are rebalanced with
 // setmaxnreg: warpgroup 0 drops to kRegsCtl, the two softmax warpgroups rise to kRegsSm.
 //   warp 0      TMA producer: Q tiles once, then K/V tiles (K0, V0, K1, V1, ...) through
@@ -111,25 +112,51 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
     volatile int* abort = &bars->abort_flag;
 
     // ---- work item ---------------------------------------------------------------------
+    // Query groups (stream, head, 256 query rows) are numbered in launch order: streams in
+    // the host's order, then head-major. Groups [0, n_full) are one item each; every later
+    // group (the tail) is cut into n_split items over contiguous KV-tile ranges, whose
+    // unnormalised partials the last of them to finish merges. Cutting only the tail fills
+    // the last wave without paying the partials' round trip on every group.
     const int item = blockIdx.x;
+    int group, split, n_parts;
+    if (item < p.n_full) {
+        group = item;
+        split = 0;
+        n_parts = 1;
+    } else {
+        const int v = item - p.n_full;
+        const int tg = v / p.n_split;
+        group = p.n_full + tg;
+        split = v - tg * p.n_split;
+        n_parts = p.n_split;
+    }
+    const int tail = group - p.n_full;                         // tail group index (n_parts > 1)
     int si = 0;
-    while (si + 1 < p.n_streams && item >= p.s[si + 1].item_begin) ++si;
+    while (si + 1 < p.n_streams && group >= p.s[si + 1].group_begin) ++si;
     const AttnStreamDesc& sd = p.s[si];
-    // items of a stream: ((head * n_split + split) * n_qpairs + pair), so CTAs launched
-    // together share one head's K/V range
-    const int local = item - sd.item_begin;
-    const int hs = local / sd.n_qpairs;
-    const int pair = local - hs * sd.n_qpairs;
-    const int head = hs / p.n_split;
-    const int split = hs - head * p.n_split;
-    const int group = sd.group_begin + head * sd.n_qpairs + pair;
+    const int local = group - sd.group_begin;
+    const int head = local / sd.n_qpairs;
+    const int pair = local - head * sd.n_qpairs;
     const int m0 = pair * (2 * kBM);
     const bool active1 = (m0 + kBM) < sd.n_q;
     const int ng = active1 ? 2 : 1;
     const int tiles_total = (sd.n_kv + kBN - 1) / kBN;
-    const int t0 = split * tiles_total / p.n_split;          // this split's KV tiles
-    const int n_tiles = (split + 1) * tiles_total / p.n_split - t0;
+    const int t0 = split * tiles_total / n_parts;            // this item's KV tiles
+    const int n_tiles = (split + 1) * tiles_total / n_parts - t0;
     const int n_loads = 2 * n_tiles;
+#ifdef FRT_DEBUG
+    // every index this item derives must lie inside the launch's extents; an item that
+    // fails records FRT_ERR_BOUNDS and exits before it touches memory (the whole CTA
+    // returns here, before any barrier or TMEM allocation)
+    if (item >= p.total_items || group < 0 || group >= p.groups_total || si >= p.n_streams ||
+        head < 0 || head >= p.heads || pair < 0 || pair >= sd.n_qpairs || n_tiles < 1 ||
+        t0 < 0 || t0 + n_tiles > tiles_total ||
+        (n_parts > 1 && (tail < 0 || tail >= p.tails_cap ||
+                         (long long)(tail + 1) * n_parts * 2 * kBM > p.part_rows_cap))) {
+        if (threadIdx.x == 0) record_status(p.status, kStatusBounds, 9, item);
+        return;
+    }
+#endif
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -541,7 +568,7 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 bulk_wait_read<0>();
             }
         };
-        if (p.n_split == 1) {
+        if (n_parts == 1) {
             if (ok) {
                 // O / l -> out
                 tc_fence_after();
@@ -560,8 +587,8 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             }
             store_out();
         } else {
-            // unnormalised partial of this split -> scratch (rows of tile (group, split, g))
-            const int prow_tile = int((size_t(group) * p.n_split + split) * 2 * kBM) + g * kBM;
+            // unnormalised partial of this split -> scratch (rows of tile (tail, split, g))
+            const int prow_tile = int((size_t(tail) * n_parts + split) * 2 * kBM) + g * kBM;
             if (ok) {
                 tc_fence_after();
 #pragma unroll 1
@@ -589,21 +616,21 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             // the last split of this query group to finish merges all partials
             named_bar_sync(1, 256);
             if (threadIdx.x == 128) {
-                const int old = atomicAdd(p.counters + group, 1);
-                const int last = (old == p.n_split - 1);
-                if (last) p.counters[group] = 0;   // every split has counted: reset for reuse
+                const int old = atomicAdd(p.counters + tail, 1);
+                const int last = (old == n_parts - 1);
+                if (last) p.counters[tail] = 0;    // every split has counted: reset for reuse
                 bars->last_split = last;
             }
             named_bar_sync(1, 256);
             if (bars->last_split) {
                 __threadfence();
                 fence_proxy_async_global();
-                const int prow0 = int(size_t(group) * p.n_split * 2 * kBM) + g * kBM;
+                const int prow0 = int(size_t(tail) * n_parts * 2 * kBM) + g * kBM;
                 float2 ml[kMaxSplit];
 #pragma unroll
                 for (int r = 0; r < kMaxSplit; ++r)
                     ml[r] = (r == split) ? make_float2(m_run, l_run)
-                            : (r < p.n_split) ? __ldcg(&p.part_ml[prow0 + r * 2 * kBM + row])
+                            : (r < n_parts) ? __ldcg(&p.part_ml[prow0 + r * 2 * kBM + row])
                                               : make_float2(-INFINITY, 0.0f);
                 float mref = -INFINITY;
 #pragma unroll
@@ -612,7 +639,7 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 float lsum = 0.0f;
 #pragma unroll
                 for (int r = 0; r < kMaxSplit; ++r) {
-                    wr[r] = (r < p.n_split) ? ex2_approx(ml[r].x - mref) : 0.0f;
+                    wr[r] = (r < n_parts) ? ex2_approx(ml[r].x - mref) : 0.0f;
                     lsum += wr[r] * ml[r].y;
                 }
                 const float w_own = ex2_approx(m_run - mref);
@@ -625,7 +652,7 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 int phase = 0;
 #pragma unroll
                 for (int r = 0; r < kMaxSplit; ++r) {
-                    if (r >= p.n_split) continue;
+                    if (r >= n_parts) continue;
                     const bool own = (r == split);
                     if (!own) {
                         const uint32_t fb = smem_u32(&bars->epi_full[g]);

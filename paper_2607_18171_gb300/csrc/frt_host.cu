@@ -184,6 +184,24 @@ enum Phase { kStart = 0, kRoped = 1, kAppended = 2 };
 
 constexpr unsigned long long kDefaultWaitLimitNs = 2000000000ull;  // 2 s per bounded wait
 
+// Guard words: kGuardBytes of kGuardByte before and after each cache buffer (one
+// allocation each), written at configure and compared by frt_stream_check_guards. A
+// kernel that wrote past either end of the ring would change them.
+constexpr size_t kGuardBytes = 256;
+constexpr unsigned char kGuardByte = 0xA7;
+#ifdef FRT_DEBUG
+constexpr bool kDebugBuild = true;
+// the debug build also keeps one chunk of slack after the rear guard (filled like the
+// guard): a write one slot past the ring that a bounds check missed would still land in
+// the library's own memory, and the guard check would report it
+constexpr bool kSlackChunk = true;
+// self-test hook: the next append targets ring slot W (one past the ring)
+int g_append_past_ring = 0;
+#else
+constexpr bool kDebugBuild = false;
+constexpr bool kSlackChunk = false;
+#endif
+
 }  // namespace
 
 struct frt_stream {
@@ -192,8 +210,11 @@ struct frt_stream {
     frt_config cfg{};
     float scale = 0.f;
     cudaStream_t cs = nullptr;
-    void* cache_k = nullptr;
+    void* cache_k = nullptr;    // ring buffers, kGuardBytes into their allocations
     void* cache_v = nullptr;
+    unsigned char* alloc_k = nullptr;   // the allocations (guard, ring, guard [, slack])
+    unsigned char* alloc_v = nullptr;
+    size_t rear_bytes = 0;              // guard (+ slack) after each ring
     size_t chunk_elems = 0;     // Nq * H * D
     float2* d_hw = nullptr;     // h/w RoPE tables
     int hw_entries = 0;
@@ -222,13 +243,16 @@ struct frt_stream {
     cudaEvent_t qkv_stop = nullptr;
     cudaEvent_t proj_start = nullptr;
     cudaEvent_t proj_stop = nullptr;
-    // split-KV scratch: partial O / (max, sum) per (query group, split), one counter per
-    // query group (zero between launches)
+    // split-KV scratch: partial O / (max, sum) rows per (tail group, split), one counter
+    // per tail group (zero between launches)
     float* part_o = nullptr;
     float2* part_ml = nullptr;
     int* counters = nullptr;
-    long long part_groups = 0;   // capacity: query groups
-    int part_splits = 1;         // capacity: splits per group
+    long long part_rows = 0;     // capacity: partial rows (256 per tail group and split)
+    long long part_tails = 0;    // capacity: tail groups (merge counters)
+    // work split of this stream's attention launch for each window fill n_valid = 1..W
+    // (index n_valid - 1), planned once at configure
+    std::vector<SplitPlan> plans;
 };
 
 namespace {
@@ -237,6 +261,10 @@ frt_status check_device_status(frt_stream_t* s) {
     if (s->status_host == nullptr) return FRT_OK;
     volatile DeviceStatus* st = s->status_host;
     int code = st->code;
+    if (code == FRT_ERR_BOUNDS)
+        return fail(FRT_ERR_BOUNDS,
+                    "device bounds check failed (block %d, role %d, at %d); reset the stream",
+                    st->block, st->role, st->where);
     if (code != 0)
         return fail(static_cast<frt_status>(code),
                     "device wait gave up (block %d, role %d, at %d); reset the stream", st->block,
@@ -269,51 +297,54 @@ void fill_rope(const frt_stream_t* s, long long c, RopeArgs& a) {
     }
 }
 
-// Split-KV factor for `groups` query groups of `tiles` KV tiles each: minimise the
-// makespan ceil(groups * s / SMs) / s, with a 2 % cost per extra split (the partial
-// round trip and merge); each split keeps at least two KV tiles.
-int choose_split(long long groups, int tiles, int max_split) {
-    const long long sms = num_sms();
-    int best = 1;
-    double best_t = double((groups + sms - 1) / sms);
-    for (int sp = 2; sp <= max_split && sp <= kMaxSplit; ++sp) {
-        if (tiles < 2 * sp) break;
-        const double t = double((groups * sp + sms - 1) / sms) / sp * (1.0 + 0.02 * (sp - 1));
-        if (t < best_t - 1e-9) {
-            best_t = t;
-            best = sp;
-        }
-    }
-    return best;
-}
-
-// Make sure s owns split-KV scratch for `groups` query groups x `splits` splits
+// Make sure s owns split-KV scratch for `rows` partial rows and `tails` merge counters
 // (allocates, synchronously, only when it must grow).
-frt_status ensure_scratch(frt_stream_t* s, long long groups, int splits) {
-    if (splits <= 1 || (groups <= s->part_groups && splits <= s->part_splits)) return FRT_OK;
+frt_status ensure_scratch(frt_stream_t* s, long long rows, long long tails) {
+    if (rows <= s->part_rows && tails <= s->part_tails) return FRT_OK;
     cudaError_t e;
     if (s->part_o && (e = cudaStreamSynchronize(s->cs)) != cudaSuccess)
         return cuda_fail(e, "sync before scratch growth");
-    const long long g = std::max(groups, s->part_groups);
-    const int sp = std::max(splits, s->part_splits);
+    const long long r = std::max(rows, s->part_rows);
+    const long long t = std::max(std::max(tails, s->part_tails), 1LL);
     if (s->part_o) cudaFree(s->part_o);
     if (s->part_ml) cudaFree(s->part_ml);
     if (s->counters) cudaFree(s->counters);
     s->part_o = nullptr;
     s->part_ml = nullptr;
     s->counters = nullptr;
-    s->part_groups = 0;
-    s->part_splits = 1;
-    const size_t rows = size_t(g) * sp * 2 * 128;
-    if ((e = cudaMalloc(&s->part_o, rows * s->head_dim * sizeof(float))) != cudaSuccess ||
-        (e = cudaMalloc(&s->part_ml, rows * sizeof(float2))) != cudaSuccess ||
-        (e = cudaMalloc(&s->counters, size_t(g) * sizeof(int))) != cudaSuccess ||
-        (e = cudaMemset(s->counters, 0, size_t(g) * sizeof(int))) != cudaSuccess ||
+    s->part_rows = 0;
+    s->part_tails = 0;
+    if ((e = cudaMalloc(&s->part_o, size_t(std::max(r, 256LL)) * s->head_dim * sizeof(float))) !=
+            cudaSuccess ||
+        (e = cudaMalloc(&s->part_ml, size_t(std::max(r, 256LL)) * sizeof(float2))) != cudaSuccess ||
+        (e = cudaMalloc(&s->counters, size_t(t) * sizeof(int))) != cudaSuccess ||
+        (e = cudaMemset(s->counters, 0, size_t(t) * sizeof(int))) != cudaSuccess ||
         (e = cudaDeviceSynchronize()) != cudaSuccess)
         return cuda_fail(e, "split-KV scratch allocation");
-    s->part_groups = g;
-    s->part_splits = sp;
+    s->part_rows = std::max(r, 256LL);
+    s->part_tails = t;
     return FRT_OK;
+}
+
+// Query groups of one stream in launch order (head-major): KV tiles and whether the
+// group has a single 128-row query tile (the ragged last group of each head).
+void stream_groups(int n_q, int heads, long long n_kv, std::vector<int>& tiles,
+                   std::vector<unsigned char>& single) {
+    const int pairs = (n_q + 255) / 256;
+    const int t = int((n_kv + 127) / 128);
+    for (int h = 0; h < heads; ++h)
+        for (int pr = 0; pr < pairs; ++pr) {
+            tiles.push_back(t);
+            single.push_back((pr * 256 + 128) >= n_q ? 1 : 0);
+        }
+}
+
+// Split-KV scratch of a launch: partial rows and merge counters.
+long long plan_rows(const SplitPlan& pl, long long groups) {
+    return pl.n_split > 1 ? (groups - pl.n_full) * pl.n_split * 256 : 0;
+}
+long long plan_tails(const SplitPlan& pl, long long groups) {
+    return pl.n_split > 1 ? groups - pl.n_full : 0;
 }
 
 int log2_exact(int x) {
@@ -338,23 +369,28 @@ frt_status attention_single(frt_stream_t* s, const void* q, void* out, bool rope
     d.n_q = s->n_q;
     d.n_kv = int(n_kv);
     d.n_qpairs = (s->n_q + 255) / 256;
-    d.item_begin = 0;
     d.group_begin = 0;
     const long long groups = (long long)d.n_qpairs * s->heads;
-    p.n_split = choose_split(groups, int((n_kv + 127) / 128), s->part_splits);
+    const SplitPlan pl = s->plans[size_t(n_valid - 1)];
+    if (plan_rows(pl, groups) > s->part_rows || plan_tails(pl, groups) > s->part_tails)
+        return fail(FRT_ERR_STATE, "split-KV scratch smaller than the configured plan");
+    p.n_full = pl.n_full;
+    p.n_split = pl.n_split;
     p.part_o = s->part_o;
     p.part_ml = s->part_ml;
     p.counters = s->counters;
+    p.groups_total = int(groups);
+    p.part_rows_cap = s->part_rows;
+    p.tails_cap = s->part_tails;
     p.n_streams = 1;
     p.heads = s->heads;
-    p.total_items = int(groups * p.n_split);
+    p.total_items = int(pl.n_full + (groups - pl.n_full) * pl.n_split);
     p.out_bf16 = out_bf16 >= 0 ? out_bf16 : (s->cfg.out_dtype == FRT_OUT_BF16);
     if ((st = make_out_map(&d.out_map, out, s->head_dim, s->heads, s->n_q, p.out_bf16 != 0)) !=
         FRT_OK)
         return st;
     if (p.n_split > 1 &&
-        (st = make_part_map(&p.part_map, s->part_o, s->head_dim,
-                            s->part_groups * s->part_splits * 256)) != FRT_OK)
+        (st = make_part_map(&p.part_map, s->part_o, s->head_dim, s->part_rows)) != FRT_OK)
         return st;
     p.scale_log2 = float(double(s->scale) * 1.4426950408889634);
     p.wait_limit_ns = s->wait_limit_ns;
@@ -375,7 +411,18 @@ frt_status append_impl(frt_stream_t* s, const void* k, const void* v, bool rope_
     frt_window_index(s->counter, s->window, &slot, &evicted, nullptr);
     AppendParams p;
     std::memset(&p, 0, sizeof(p));
-    const size_t off = size_t(slot) * s->chunk_elems;
+    size_t off = size_t(slot) * s->chunk_elems;
+#ifdef FRT_DEBUG
+    if (g_append_past_ring) {   // self-test: aim one slot past the ring
+        off = size_t(s->window) * s->chunk_elems;
+        g_append_past_ring = 0;
+    }
+#endif
+    const size_t cache_bytes = size_t(s->window) * s->chunk_elems * 2;
+    p.k_lo = s->cache_k;
+    p.k_hi = static_cast<const uint8_t*>(s->cache_k) + cache_bytes;
+    p.v_lo = s->cache_v;
+    p.v_hi = static_cast<const uint8_t*>(s->cache_v) + cache_bytes;
     p.k_src = static_cast<const uint4*>(k);
     p.v_src = static_cast<const uint4*>(v);
     p.k_dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(s->cache_k) + off);
@@ -401,8 +448,9 @@ frt_status append_impl(frt_stream_t* s, const void* k, const void* v, bool rope_
 }
 
 void free_device(frt_stream_t* s) {
-    if (s->cache_k) cudaFree(s->cache_k);
-    if (s->cache_v) cudaFree(s->cache_v);
+    if (s->alloc_k) cudaFree(s->alloc_k);
+    if (s->alloc_v) cudaFree(s->alloc_v);
+    s->alloc_k = s->alloc_v = nullptr;
     if (s->d_hw) cudaFree(s->d_hw);
     if (s->stage) cudaFree(s->stage);
     if (s->status_host) cudaFreeHost(s->status_host);
@@ -425,8 +473,8 @@ void free_device(frt_stream_t* s) {
     s->part_o = nullptr;
     s->part_ml = nullptr;
     s->counters = nullptr;
-    s->part_groups = 0;
-    s->part_splits = 1;
+    s->part_rows = 0;
+    s->part_tails = 0;
     s->cache_k = s->cache_v = nullptr;
     s->d_hw = nullptr;
     s->stage = nullptr;
@@ -450,6 +498,7 @@ const char* frt_status_string(frt_status st) {
         case FRT_ERR_CUDA: return "FRT_ERR_CUDA";
         case FRT_ERR_UNSUPPORTED: return "FRT_ERR_UNSUPPORTED";
         case FRT_ERR_TIMEOUT: return "FRT_ERR_TIMEOUT";
+        case FRT_ERR_BOUNDS: return "FRT_ERR_BOUNDS";
     }
     return "FRT_ERR_UNKNOWN";
 }
@@ -545,11 +594,22 @@ frt_status frt_stream_configure(frt_stream_t* s, const frt_config* cfg) {
     cudaError_t e;
     const size_t cache_bytes = size_t(s->window) * s->chunk_elems * 2;
     if (!s->cache_k) {
-        if ((e = cudaMalloc(&s->cache_k, cache_bytes)) != cudaSuccess ||
-            (e = cudaMalloc(&s->cache_v, cache_bytes)) != cudaSuccess) {
+        s->rear_bytes = kGuardBytes + (kSlackChunk ? s->chunk_elems * 2 : 0);
+        const size_t total = kGuardBytes + cache_bytes + s->rear_bytes;
+        if ((e = cudaMalloc(reinterpret_cast<void**>(&s->alloc_k), total)) != cudaSuccess ||
+            (e = cudaMalloc(reinterpret_cast<void**>(&s->alloc_v), total)) != cudaSuccess) {
             free_device(s);
             return cuda_fail(e, "cache allocation");
         }
+        s->cache_k = s->alloc_k + kGuardBytes;
+        s->cache_v = s->alloc_v + kGuardBytes;
+        for (unsigned char* a : {s->alloc_k, s->alloc_v})
+            if ((e = cudaMemset(a, kGuardByte, kGuardBytes)) != cudaSuccess ||
+                (e = cudaMemset(a + kGuardBytes + cache_bytes, kGuardByte, s->rear_bytes)) !=
+                    cudaSuccess) {
+                free_device(s);
+                return cuda_fail(e, "guard words");
+            }
     }
     if (!s->status_host) {
         if ((e = cudaHostAlloc(reinterpret_cast<void**>(&s->status_host), sizeof(DeviceStatus),
@@ -590,10 +650,21 @@ frt_status frt_stream_configure(frt_stream_t* s, const frt_config* cfg) {
         return cuda_fail(e, "rope table upload");
     s->hw_entries = int(hw.size());
     {
-        // split-KV scratch for the steady-state (full window) launch of this stream
+        // the work split of every window fill, and split-KV scratch for all of them
         const long long groups = (long long)((s->n_q + 255) / 256) * s->heads;
-        const int tiles = int(((long long)s->window * s->n_q + 127) / 128);
-        frt_status st = ensure_scratch(s, groups, choose_split(groups, tiles, kMaxSplit));
+        s->plans.clear();
+        long long rows = 0, tails = 0;
+        for (int nv = 1; nv <= s->window; ++nv) {
+            std::vector<int> tiles;
+            std::vector<unsigned char> single;
+            stream_groups(s->n_q, s->heads, (long long)nv * s->n_q, tiles, single);
+            const SplitPlan pl = plan_attention(tiles.data(), single.data(), int(groups),
+                                                num_sms(), kMaxSplit, -1, -1);
+            s->plans.push_back(pl);
+            rows = std::max(rows, plan_rows(pl, groups));
+            tails = std::max(tails, plan_tails(pl, groups));
+        }
+        frt_status st = ensure_scratch(s, rows, tails);
         if (st != FRT_OK) {
             free_device(s);
             return st;
@@ -604,7 +675,7 @@ frt_status frt_stream_configure(frt_stream_t* s, const frt_config* cfg) {
     if ((e = cudaMemset(s->cache_k, 0, cache_bytes)) != cudaSuccess ||
         (e = cudaMemset(s->cache_v, 0, cache_bytes)) != cudaSuccess ||
         (s->counters &&
-         (e = cudaMemset(s->counters, 0, size_t(s->part_groups) * sizeof(int))) != cudaSuccess))
+         (e = cudaMemset(s->counters, 0, size_t(s->part_tails) * sizeof(int))) != cudaSuccess))
         return cuda_fail(e, "cache clear");
     if ((e = cudaDeviceSynchronize()) != cudaSuccess) return cuda_fail(e, "configure sync");
     s->counter = 0;
@@ -856,6 +927,23 @@ frt_status frt_chunk_step_host(frt_stream_t* s, const void* q_host, const void* 
     return FRT_OK;
 }
 
+frt_status frt_attention_plan(int n, const int* n_q, const long long* n_kv, int heads, int sms,
+                              int* n_full, int* n_split) {
+    if (n < 1 || !n_q || !n_kv || heads < 1 || !n_full || !n_split)
+        return fail(FRT_ERR_INVALID_ARG, "need n >= 1, heads >= 1 and non-NULL arrays");
+    std::vector<int> tiles;
+    std::vector<unsigned char> single;
+    for (int i = 0; i < n; ++i) {
+        if (n_q[i] < 1 || n_kv[i] < 1) return fail(FRT_ERR_INVALID_ARG, "sizes must be >= 1");
+        stream_groups(n_q[i], heads, n_kv[i], tiles, single);
+    }
+    const SplitPlan pl = plan_attention(tiles.data(), single.data(), int(tiles.size()),
+                                        sms > 0 ? sms : num_sms(), kMaxSplit, -1, -1);
+    *n_full = pl.n_full;
+    *n_split = pl.n_split;
+    return FRT_OK;
+}
+
 frt_status frt_chunk_attention_batched(frt_stream_t* const* streams, int n, const void* const* q,
                                        void* const* out) {
     if (!streams || !q || !out || n < 1 || n > kMaxBatchStreams)
@@ -886,27 +974,36 @@ frt_status frt_chunk_attention_batched(frt_stream_t* const* streams, int n, cons
     auto* p = new (std::nothrow) AttnParams<kMaxBatchStreams>();
     if (!p) return fail(FRT_ERR_OOM, "host allocation failed");
     std::memset(p, 0, sizeof(*p));
-    long long groups_total = 0;
-    int min_tiles = 1 << 30;
-    for (int i = 0; i < n; ++i) {
-        groups_total += (long long)((streams[i]->n_q + 255) / 256) * streams[i]->heads;
-        min_tiles = std::min(min_tiles, int((n_kv(i) + 127) / 128));
+    // query groups in launch order (streams longest KV first, then head-major) and the
+    // work split of the launch
+    std::vector<int> tiles;
+    std::vector<unsigned char> single;
+    for (int oi = 0; oi < n; ++oi) {
+        const int i = order[oi];
+        stream_groups(streams[i]->n_q, streams[i]->heads, n_kv(i), tiles, single);
     }
-    const int n_split = choose_split(groups_total, min_tiles, kMaxSplit);
-    if ((st = ensure_scratch(s0, groups_total, n_split)) != FRT_OK) {
+    const long long groups_total = (long long)tiles.size();
+    const SplitPlan pl = plan_attention(tiles.data(), single.data(), int(groups_total), num_sms(),
+                                        kMaxSplit, -1, -1);
+    if ((st = ensure_scratch(s0, plan_rows(pl, groups_total), plan_tails(pl, groups_total))) !=
+        FRT_OK) {
         delete p;
         return st;
     }
-    p->n_split = n_split;
-    if (n_split > 1 && (st = make_part_map(&p->part_map, s0->part_o, s0->head_dim,
-                                           s0->part_groups * s0->part_splits * 256)) != FRT_OK) {
+    p->n_full = pl.n_full;
+    p->n_split = pl.n_split;
+    if (pl.n_split > 1 &&
+        (st = make_part_map(&p->part_map, s0->part_o, s0->head_dim, s0->part_rows)) != FRT_OK) {
         delete p;
         return st;
     }
     p->part_o = s0->part_o;
     p->part_ml = s0->part_ml;
     p->counters = s0->counters;
-    int items = 0, groups = 0;
+    p->groups_total = int(groups_total);
+    p->part_rows_cap = s0->part_rows;
+    p->tails_cap = s0->part_tails;
+    int groups = 0;
     for (int oi = 0; oi < n; ++oi) {
         const int i = order[oi];
         frt_stream_t* s = streams[i];
@@ -927,11 +1024,10 @@ frt_status frt_chunk_attention_batched(frt_stream_t* const* streams, int n, cons
         d.n_q = s->n_q;
         d.n_kv = int(nkv);
         d.n_qpairs = (s->n_q + 255) / 256;
-        d.item_begin = items;
         d.group_begin = groups;
-        items += d.n_qpairs * s->heads * n_split;
         groups += d.n_qpairs * s->heads;
     }
+    const int items = int(pl.n_full + (groups_total - pl.n_full) * pl.n_split);
     p->n_streams = n;
     p->heads = s0->heads;
     p->total_items = items;
@@ -969,7 +1065,10 @@ frt_status frt_stream_sync(frt_stream_t* s) {
     if (e == cudaSuccess && s->cp_in) e = cudaStreamSynchronize(s->cp_in);
     if (e == cudaSuccess && s->cp_out) e = cudaStreamSynchronize(s->cp_out);
     if (e != cudaSuccess) return cuda_fail(e, "stream sync");
-    return check_device_status(s);
+    frt_status st = check_device_status(s);
+    // the debug build also compares the guard words around the cache at every sync
+    if (st == FRT_OK && kDebugBuild) st = frt_stream_check_guards(s);
+    return st;
 }
 
 frt_status frt_stream_reset(frt_stream_t* s) {
@@ -984,7 +1083,7 @@ frt_status frt_stream_reset(frt_stream_t* s) {
     // reset) may have left some of them counted, which would elect a merging split early
     if ((e = cudaMemsetAsync(s->cache_k, 0, cache_bytes, s->cs)) != cudaSuccess ||
         (e = cudaMemsetAsync(s->cache_v, 0, cache_bytes, s->cs)) != cudaSuccess ||
-        (s->counters && (e = cudaMemsetAsync(s->counters, 0, size_t(s->part_groups) * sizeof(int),
+        (s->counters && (e = cudaMemsetAsync(s->counters, 0, size_t(s->part_tails) * sizeof(int),
                                              s->cs)) != cudaSuccess) ||
         (e = cudaStreamSynchronize(s->cs)) != cudaSuccess)
         return cuda_fail(e, "cache clear");
@@ -1031,6 +1130,68 @@ frt_status frt_stream_set_append_events(frt_stream_t* s, void* start_event, void
         return fail(FRT_ERR_INVALID_ARG, "give both events or neither");
     s->app_start = static_cast<cudaEvent_t>(start_event);
     s->app_stop = static_cast<cudaEvent_t>(stop_event);
+    return FRT_OK;
+}
+
+int frt_debug_build(void) { return kDebugBuild ? 1 : 0; }
+
+frt_status frt_stream_check_guards(frt_stream_t* s) {
+    if (!s) return fail(FRT_ERR_INVALID_ARG, "NULL stream handle");
+    if (!s->configured || !s->alloc_k) return fail(FRT_ERR_STATE, "stream not configured");
+    cudaError_t e = cudaStreamSynchronize(s->cs);
+    if (e != cudaSuccess) return cuda_fail(e, "stream sync");
+    const size_t cache_bytes = size_t(s->window) * s->chunk_elems * 2;
+    std::vector<unsigned char> h(std::max(kGuardBytes, s->rear_bytes));
+    const char* names[2] = {"K", "V"};
+    unsigned char* allocs[2] = {s->alloc_k, s->alloc_v};
+    for (int b = 0; b < 2; ++b) {
+        const struct { size_t off, len; const char* where; } parts[2] = {
+            {0, kGuardBytes, "before"}, {kGuardBytes + cache_bytes, s->rear_bytes, "after"}};
+        for (const auto& pt : parts) {
+            if ((e = cudaMemcpy(h.data(), allocs[b] + pt.off, pt.len, cudaMemcpyDeviceToHost)) !=
+                cudaSuccess)
+                return cuda_fail(e, "guard read");
+            for (size_t i = 0; i < pt.len; ++i)
+                if (h[i] != kGuardByte)
+                    return fail(FRT_ERR_BOUNDS, "guard word %s the %s cache overwritten (byte %zu)",
+                                pt.where, names[b], i);
+        }
+    }
+    return FRT_OK;
+}
+
+frt_status frt_stream_save(frt_stream_t* s, void* k_dst, void* v_dst, long long* counter) {
+    frt_status st = require_configured(s);
+    if (st != FRT_OK) return st;
+    if (!k_dst || !v_dst || !counter) return fail(FRT_ERR_INVALID_ARG, "NULL destination");
+    if (s->phase == kRoped) return fail(FRT_ERR_STATE, "a chunk is half done (rope without append)");
+    const size_t cache_bytes = size_t(s->window) * s->chunk_elems * 2;
+    cudaError_t e;
+    if ((e = cudaMemcpyAsync(k_dst, s->cache_k, cache_bytes, cudaMemcpyDefault, s->cs)) !=
+            cudaSuccess ||
+        (e = cudaMemcpyAsync(v_dst, s->cache_v, cache_bytes, cudaMemcpyDefault, s->cs)) !=
+            cudaSuccess)
+        return cuda_fail(e, "snapshot copy");
+    *counter = s->counter;
+    return FRT_OK;
+}
+
+frt_status frt_stream_restore(frt_stream_t* s, const void* k_src, const void* v_src,
+                              long long counter) {
+    frt_status st = require_configured(s);
+    if (st != FRT_OK) return st;
+    if (!k_src || !v_src) return fail(FRT_ERR_INVALID_ARG, "NULL source");
+    if (counter < 0) return fail(FRT_ERR_INVALID_ARG, "counter must be >= 0");
+    const size_t cache_bytes = size_t(s->window) * s->chunk_elems * 2;
+    cudaError_t e;
+    if ((e = cudaMemcpyAsync(s->cache_k, k_src, cache_bytes, cudaMemcpyDefault, s->cs)) !=
+            cudaSuccess ||
+        (e = cudaMemcpyAsync(s->cache_v, v_src, cache_bytes, cudaMemcpyDefault, s->cs)) !=
+            cudaSuccess)
+        return cuda_fail(e, "restore copy");
+    s->counter = counter;
+    s->phase = kStart;
+    s->last_q = s->last_k = s->last_v = nullptr;
     return FRT_OK;
 }
 
@@ -1130,3 +1291,25 @@ void frt_steps_destroy(frt_steps_t* g) {
 }
 
 }  // extern "C"
+
+extern "C" frt_status frt_selftest_append_past_ring(void) {
+#ifdef FRT_DEBUG
+    g_append_past_ring = 1;
+    return FRT_OK;
+#else
+    return fail(FRT_ERR_UNSUPPORTED, "only the FRT_DEBUG build has this hook");
+#endif
+}
+
+extern "C" frt_status frt_selftest_poke_guard(frt_stream_t* s, int which) {
+    if (!s || !s->configured || !s->alloc_k) return fail(FRT_ERR_STATE, "stream not configured");
+    if (which < 0 || which > 3) return fail(FRT_ERR_INVALID_ARG, "which in 0..3");
+    const size_t cache_bytes = size_t(s->window) * s->chunk_elems * 2;
+    unsigned char* a = (which & 1) ? s->alloc_v : s->alloc_k;
+    unsigned char* at = (which & 2) ? a + kGuardBytes + cache_bytes : a + kGuardBytes - 1;
+    cudaError_t e = cudaStreamSynchronize(s->cs);
+    if (e == cudaSuccess) e = cudaMemset(at, 0x00, 1);
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return cuda_fail(e, "guard poke");
+    return FRT_OK;
+}

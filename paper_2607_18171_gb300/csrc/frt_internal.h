@@ -13,11 +13,16 @@ constexpr int kMaxBatchStreams = 32;
 // Largest split-KV factor (KV ranges per query group).
 constexpr int kMaxSplit = 4;
 
+// Status codes the kernels record (frt_status values).
+constexpr int kStatusTimeout = 6;   // FRT_ERR_TIMEOUT
+constexpr int kStatusBounds = 7;    // FRT_ERR_BOUNDS (FRT_DEBUG builds)
+
 // Device status block (host-mapped pinned memory): the first device error wins.
 struct DeviceStatus {
     int code;      // 0 = ok, else an frt_status value
     int block;     // blockIdx.x of the CTA that reported it
-    int role;      // 0 producer, 1 mma issuer, 2-3 softmax groups, 4 observer (attention)
+    int role;      // 0 producer, 1 mma issuer, 2-3 softmax groups, 4 observer, 9 item
+                   // check (attention); 100+ append / RoPE kernel
     int where;     // loop iteration or barrier id
 };
 
@@ -83,8 +88,7 @@ struct AttnStreamDesc {
     int n_q;
     int n_kv;
     int n_qpairs;        // ceil(Nq / 256): query groups per head
-    int item_begin;      // first work item of this stream
-    int group_begin;     // first query group (head, 256 rows) of this stream
+    int group_begin;     // first query group (head, 256 rows) of this stream, launch order
 };
 
 template <int MAXS>
@@ -95,16 +99,22 @@ struct AttnParams {
     int total_items;
     int out_bf16;
     float scale_log2;            // sm_scale * log2(e)
-    // Split-KV: each query group's KV tiles are cut into n_split contiguous ranges
-    // processed by separate CTAs; each writes an unnormalised partial (O, running max,
-    // row sum) and the last to finish merges them. n_split == 1 uses none of these.
+    // Split-KV of the tail: query groups [0, n_full) run whole, one item each; each later
+    // group (tail group t = group - n_full) has its KV tiles cut into n_split contiguous
+    // ranges processed by separate CTAs; each writes an unnormalised partial (O, running
+    // max, row sum) and the last to finish merges them. n_full == groups uses none of these.
+    int n_full;
     int n_split;
-    CUtensorMap part_map;        // 2D (D, groups * n_split * 256) fp32 over part_o, box (32, 128)
-    float* part_o;               // [groups * n_split][2][128][D] fp32
-    float2* part_ml;             // [groups * n_split][2][128] (max in log2 units, sum)
-    int* counters;               // [groups], zero between launches
+    CUtensorMap part_map;        // 2D (D, tail groups * n_split * 256) fp32 over part_o, box (32, 128)
+    float* part_o;               // [tail groups * n_split][2][128][D] fp32
+    float2* part_ml;             // [tail groups * n_split][2][128] (max in log2 units, sum)
+    int* counters;               // [tail groups], zero between launches
     unsigned long long wait_limit_ns;
     DeviceStatus* status;
+    // extents the FRT_DEBUG build checks every work item's indices against
+    int groups_total;            // query groups of the launch
+    long long part_rows_cap;     // partial rows the scratch holds
+    long long tails_cap;         // merge counters the scratch holds
     RopeArgs rope;               // RoPE-Q prologue (single-stream fused path only)
 };
 
@@ -118,6 +128,10 @@ struct AppendParams {
     int vec_per_head_log2;  // log2(D / 8)
     int rope;               // rotate K on the way
     DeviceStatus* status;   // bounded-wait timeouts are recorded here
+    const void* k_lo;       // the ring buffers' extents [lo, hi): the FRT_DEBUG build checks
+    const void* k_hi;       // every store against them
+    const void* v_lo;
+    const void* v_hi;
     RopeArgs ra;
 };
 
@@ -162,6 +176,32 @@ struct GemmParams {
     DeviceStatus* status;
     RopeArgs ra;
 };
+
+// Work split of one attention launch: query groups [0, n_full) (launch order) run whole,
+// each later group is cut into n_split KV parts whose partials are merged.
+struct SplitPlan {
+    int n_full = 0;
+    int n_split = 1;
+};
+// Plans a launch over `groups` query groups with tiles[g] KV tiles each (single[g] != 0:
+// one 128-row query tile) on `sms` SMs: the tail split whose simulated list schedule ends
+// first. At most max_split parts, every part at least two KV tiles; max_rows / max_tails
+// bound the split-KV scratch (partial rows, merge counters; negative: unbounded).
+SplitPlan plan_attention(const int* tiles, const unsigned char* single, int groups, int sms,
+                         int max_split, long long max_rows, long long max_tails);
+
+// Record `code` in the status block unless an earlier error is there (first one wins).
+__device__ __forceinline__ void record_status(DeviceStatus* st, int code, int role, int where) {
+    if (st == nullptr) return;
+    volatile DeviceStatus* s = st;
+    if (s->code == 0) {
+        s->block = blockIdx.x;
+        s->role = role;
+        s->where = where;
+        __threadfence_system();
+        s->code = code;
+    }
+}
 
 // Kernel launchers (defined in the .cu files).
 cudaError_t launch_gemm(GemmParams p, cudaStream_t st);

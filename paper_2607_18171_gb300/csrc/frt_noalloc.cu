@@ -221,7 +221,11 @@ extern "C" frt_status frt_chunk_attention_noalloc(const void* q, const void* k, 
     d.n_qpairs = n_qpairs;
     p.n_streams = 1;
     p.heads = heads;
+    p.n_full = 0;          // every group is cut into `split` parts (split 1: run whole)
     p.n_split = split;
+    p.groups_total = int(groups);
+    p.part_rows_cap = (long long)cap_rows;
+    p.tails_cap = kMaxGroups;
     p.total_items = int(groups * split);
     p.part_o = part_o;
     p.part_ml = part_ml;

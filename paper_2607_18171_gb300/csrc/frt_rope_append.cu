@@ -34,6 +34,10 @@ struct StagedParams {
     int vec_per_head_log2;   // log2(head_dim / 8)
     int tok_per_block;       // tokens per stage
     int stages;              // ring depth (<= kMaxStages)
+    const uint8_t* a_lo;     // destination extents [lo, hi) checked by the FRT_DEBUG build
+    const uint8_t* a_hi;
+    const uint8_t* b_lo;
+    const uint8_t* b_hi;
     unsigned long long wait_limit_ns;
     DeviceStatus* status;
     RopeArgs ra;
@@ -102,8 +106,18 @@ __global__ void __launch_bounds__(kThreads, 1) staged_rows_kernel(const __grid_c
                 }
                 const int tok0 = (blockIdx.x + i * gridDim.x) * T;
                 const uint32_t bytes = uint32_t(min(T, p.n_tok - tok0)) * p.row_bytes;
-                bulk_store(p.a_dst + size_t(tok0) * p.row_bytes, ring0 + s * 2 * half, bytes);
-                bulk_store(p.b_dst + size_t(tok0) * p.row_bytes, ring0 + s * 2 * half + half, bytes);
+                uint8_t* ad = p.a_dst + size_t(tok0) * p.row_bytes;
+                uint8_t* bd = p.b_dst + size_t(tok0) * p.row_bytes;
+#ifdef FRT_DEBUG
+                // a store outside its destination's extent is recorded and skipped
+                if (ad < p.a_lo || ad + bytes > p.a_hi || bd < p.b_lo || bd + bytes > p.b_hi) {
+                    record_status(p.status, kStatusBounds, 102, tok0);
+                } else
+#endif
+                {
+                    bulk_store(ad, ring0 + s * 2 * half, bytes);
+                    bulk_store(bd, ring0 + s * 2 * half + half, bytes);
+                }
                 bulk_commit();
                 ++stored;
                 // block i + kStages - 1 reuses the stage of block i - 1: its stores must
@@ -208,6 +222,10 @@ cudaError_t launch_kv_append(const AppendParams& p, cudaStream_t st) {
     sp.b_dst = reinterpret_cast<uint8_t*>(p.v_dst);
     sp.rot_a = p.rope;
     sp.rot_b = 0;
+    sp.a_lo = static_cast<const uint8_t*>(p.k_lo);
+    sp.a_hi = static_cast<const uint8_t*>(p.k_hi);
+    sp.b_lo = static_cast<const uint8_t*>(p.v_lo);
+    sp.b_hi = static_cast<const uint8_t*>(p.v_hi);
     sp.n_tok = p.n_tok;
     sp.row_bytes = p.vec_per_tok * 16;
     sp.vec_per_tok = p.vec_per_tok;
@@ -226,6 +244,10 @@ cudaError_t launch_rope_qk(const RopeParams& p, cudaStream_t st) {
     sp.b_dst = reinterpret_cast<uint8_t*>(p.k);
     sp.rot_a = 1;
     sp.rot_b = 1;
+    sp.a_lo = sp.a_dst;
+    sp.a_hi = sp.a_dst + size_t(p.n_tok) * p.vec_per_tok * 16;
+    sp.b_lo = sp.b_dst;
+    sp.b_hi = sp.b_dst + size_t(p.n_tok) * p.vec_per_tok * 16;
     sp.n_tok = p.n_tok;
     sp.row_bytes = p.vec_per_tok * 16;
     sp.vec_per_tok = p.vec_per_tok;

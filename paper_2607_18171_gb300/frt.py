@@ -13,11 +13,15 @@ import os
 import torch
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_HERE, "libfrt.so")
+# FRT_LIBRARY=debug loads the FRT_DEBUG build (bounds-checking kernels, guard words checked
+# at every sync); built by _build.build(debug=True)
+LIB_PATH = os.path.join(_HERE, "libfrt_debug.so" if os.environ.get("FRT_LIBRARY") == "debug"
+                        else "libfrt.so")
 
 FRT_OK = 0
 STATUS_NAMES = {0: "FRT_OK", 1: "FRT_ERR_INVALID_ARG", 2: "FRT_ERR_STATE", 3: "FRT_ERR_OOM",
-                4: "FRT_ERR_CUDA", 5: "FRT_ERR_UNSUPPORTED", 6: "FRT_ERR_TIMEOUT"}
+                4: "FRT_ERR_CUDA", 5: "FRT_ERR_UNSUPPORTED", 6: "FRT_ERR_TIMEOUT",
+                7: "FRT_ERR_BOUNDS"}
 OUT_F32, OUT_BF16 = 0, 1
 
 
@@ -63,6 +67,12 @@ def lib() -> ctypes.CDLL:
         "frt_stream_destroy": (None, [P]),
         "frt_stream_chunk_counter": (LL, [P]),
         "frt_stream_cache": (I, [P, ctypes.POINTER(P), ctypes.POINTER(P), ctypes.POINTER(LL)]),
+        "frt_stream_save": (I, [P, P, P, ctypes.POINTER(LL)]),
+        "frt_stream_restore": (I, [P, P, P, LL]),
+        "frt_stream_check_guards": (I, [P]),
+        "frt_debug_build": (I, []),
+        "frt_selftest_append_past_ring": (I, []),
+        "frt_selftest_poke_guard": (I, [P, I]),
         "frt_stream_set_attention_events": (I, [P, P, P]),
         "frt_stream_set_append_events": (I, [P, P, P]),
         "frt_chunk_attention_noalloc": (I, [P, P, P, P, I, I, I, I, D, I, P, P]),
@@ -77,6 +87,8 @@ def lib() -> ctypes.CDLL:
         "frt_conv_destroy": (None, [P]),
         "frt_gemm_bf16": (I, [P, P, P, I, I, I, I, I, P, P]),
         "frt_gemm_plan": (I, [I, I, I, I, ctypes.POINTER(I), ctypes.POINTER(I)]),
+        "frt_attention_plan": (I, [I, ctypes.POINTER(I), ctypes.POINTER(LL), I, I,
+                                   ctypes.POINTER(I), ctypes.POINTER(I)]),
         "frt_stream_set_block_events": (I, [P, P, P, P, P]),
         "frt_window_index": (I, [LL, I, ctypes.POINTER(I), ctypes.POINTER(LL),
                                  ctypes.POINTER(I)]),
@@ -160,8 +172,13 @@ class Stream:
     # -- lifetime --------------------------------------------------------------------
     def close(self) -> None:
         if getattr(self, "_h", None):
-            lib().frt_stream_destroy(self._h)
-            self._h = None
+            h, self._h = self._h, None
+            # the debug build compares the cache's guard words before every release
+            rc = lib().frt_stream_check_guards(h) if lib().frt_debug_build() else FRT_OK
+            msg = lib().frt_last_error().decode() if rc != FRT_OK else ""
+            lib().frt_stream_destroy(h)
+            if rc not in (FRT_OK, 2):   # 2: never configured
+                raise FrtError(rc, msg)
 
     def __del__(self):  # pragma: no cover - best effort
         try:
@@ -262,6 +279,28 @@ class Stream:
         _check(lib().frt_stream_set_append_events(
             self._h, None if start is None else ctypes.c_void_p(start.cuda_event),
             None if stop is None else ctypes.c_void_p(stop.cuda_event)))
+
+    def check_guards(self) -> None:
+        """Wait for the stream and compare the guard words around its KV cache."""
+        _check(lib().frt_stream_check_guards(self._h))
+
+    def save(self):
+        """Snapshot of the persistent state: (k, v, counter), k and v device copies of
+        the whole ring. Complete once sync() returns."""
+        rows = self.window * self.n_q
+        k = torch.empty((rows, self.heads, self.head_dim), dtype=torch.bfloat16, device="cuda")
+        v = torch.empty_like(k)
+        c = ctypes.c_longlong()
+        _check(lib().frt_stream_save(self._h, _ptr(k), _ptr(v), ctypes.byref(c)))
+        return k, v, c.value
+
+    def restore(self, k: torch.Tensor, v: torch.Tensor, counter: int) -> None:
+        """Continue from a snapshot taken by save() (of this or another stream of the same
+        shape)."""
+        rows = self.window * self.n_q
+        _bf16_dev(k, (rows, self.heads, self.head_dim), "k")
+        _bf16_dev(v, (rows, self.heads, self.head_dim), "v")
+        _check(lib().frt_stream_restore(self._h, _ptr(k), _ptr(v), counter))
 
     def cache(self):
         """(k_cache, v_cache) device tensors viewing the stream's ring buffer
@@ -434,6 +473,18 @@ def gemm_plan(M: int, N: int, qkv: bool = False, d: int = 0) -> tuple[int, int]:
     bn, ctas = ctypes.c_int(), ctypes.c_int()
     _check(lib().frt_gemm_plan(M, N, 1 if qkv else 0, d, ctypes.byref(bn), ctypes.byref(ctas)))
     return bn.value, ctas.value
+
+
+def attention_plan(n_q, n_kv, heads: int, sms: int = 0) -> tuple[int, int]:
+    """(n_full, n_split) of one attention launch over streams with n_q[i] queries and
+    n_kv[i] valid keys (launch order): query groups [0, n_full) run whole, later ones are
+    cut into n_split KV parts."""
+    n = len(n_q)
+    a = (ctypes.c_int * n)(*n_q)
+    b = (ctypes.c_longlong * n)(*n_kv)
+    nf, ns = ctypes.c_int(), ctypes.c_int()
+    _check(lib().frt_attention_plan(n, a, b, heads, sms, ctypes.byref(nf), ctypes.byref(ns)))
+    return nf.value, ns.value
 
 
 def gemm_bf16(a: torch.Tensor, b: torch.Tensor, c: torch.Tensor,

@@ -175,3 +175,74 @@ def test_gemm_plan_is_host_only_and_checks_arguments(frt):
     for args in ((0, 16, False, 0), (16, 0, False, 0), (16, 48, True, 0)):
         with pytest.raises(frt.FrtError):
             frt.gemm_plan(*args)
+
+
+def _groups(n_q, n_kv, heads):
+    """Query groups of one stream in launch order: (KV tiles, one query tile?)."""
+    pairs = -(-n_q // 256)
+    return [(-(-n_kv // 128), pr * 256 + 128 >= n_q) for _ in range(heads) for pr in range(pairs)]
+
+
+def _list_schedule(items, sms):
+    """Makespan of handing `items` (costs, in order) to the SM that frees first."""
+    import heapq
+    free = [0.0] * sms
+    for c in items:
+        t = heapq.heappop(free) + c
+        heapq.heappush(free, t)
+    return max(free)
+
+
+def _plan_items(groups, n_full, n_split):
+    # the planner's cost model: 7 KV steps per item, 1 more per split item, 0.6 per
+    # KV step of a one-tile group
+    out = []
+    for g, (tiles, single) in enumerate(groups):
+        w = 0.6 if single else 1.0
+        if g < n_full:
+            out.append(7.0 + tiles * w)
+        else:
+            out += [8.0 + ((s + 1) * tiles // n_split - s * tiles // n_split) * w
+                    for s in range(n_split)]
+    return out
+
+
+@pytest.mark.parametrize("n_q,n_kv,heads", [(4680, 32760, 12), (4680, 32760, 40),
+                                            (10800, 64800, 40), (4680, 4680, 40),
+                                            (256, 5120, 2), (48, 144, 2), (390, 128, 3)])
+def test_attention_plan_is_valid_and_beats_whole_and_uniform_splits(frt, n_q, n_kv, heads):
+    sms = 152
+    n_full, n_split = frt.attention_plan([n_q], [n_kv], heads, sms)
+    groups = _groups(n_q, n_kv, heads)
+    G = len(groups)
+    assert 0 <= n_full <= G and 1 <= n_split <= 4
+    if n_split == 1:
+        assert n_full == G
+    else:
+        assert n_full < G
+        assert all(t >= 2 * n_split for t, _ in groups[n_full:])   # parts of >= 2 KV tiles
+    best = _list_schedule(_plan_items(groups, n_full, n_split), sms)
+    assert best <= _list_schedule(_plan_items(groups, G, 1), sms) + 1e-9
+    for s in range(2, 5):
+        if all(t >= 2 * s for t, _ in groups):
+            assert best <= _list_schedule(_plan_items(groups, 0, s), sms) + 1e-9
+
+
+def test_attention_plan_worked_examples(frt):
+    # 1.3B shape: 12 heads x 19 query groups = 228 groups of 256 KV tiles on 152 SMs. One
+    # whole wave of 152 groups, then the other 76 cut in two: the second wave is 152
+    # halves instead of 76 whole groups next to 76 idle SMs
+    assert frt.attention_plan([4680], [32760], 12, 152) == (152, 2)
+    # 14B shape: 760 groups = exactly 5 waves: nothing to cut
+    assert frt.attention_plan([4680], [32760], 40, 152) == (760, 1)
+    # one KV tile per group: nothing can be cut
+    assert frt.attention_plan([4680], [100], 12, 152) == (228, 1)
+    # two groups on 152 SMs: both cut as finely as allowed
+    assert frt.attention_plan([256], [128 * 40], 2, 152) == (0, 4)
+
+
+def test_attention_plan_checks_arguments(frt):
+    with pytest.raises(frt.FrtError):
+        frt.attention_plan([0], [10], 2)
+    with pytest.raises(frt.FrtError):
+        frt.attention_plan([10], [10], 0)
