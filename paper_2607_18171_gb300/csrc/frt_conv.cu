@@ -19,10 +19,13 @@
 // memory addresses, so any whole-row start is valid once the halo sits at a 1024-byte
 // boundary. This brings each input pixel into the SM about 1.4 times per temporal tap
 // and channel block instead of kh x kw times. B is the tap's [Cout, Cin] weight slice.
-// Persistent kernel, 224 threads:
+// Persistent kernel, 256 threads:
 //   warp 0      TMA producer of the halo ring;
 //   warp 6      TMA producer of the weight ring (one slice per spatial tap);
-//   warp 1      TMEM allocator + single-thread tcgen05.mma issuer (M 128, N = BN, K 16);
+//   warp 1      TMEM allocator + tcgen05.mma issuer (M 128, N = BN, K 16): a converged
+//               warp whose lane 0 issues; it touches no mbarrier in its loops;
+//   warp 7      observer: waits on the halo, weight and accumulator barriers in the
+//               issuer's order and hands each off to it through a named barrier;
 //   warps 2-5   epilogue: one thread per output pixel of the tile adds the bias and
 //               writes its 128-byte slice of each column unit (32 fp32 or 64 bf16
 //               channels) into a 128-byte-swizzled staging slab, which one TMA tensor
@@ -48,7 +51,10 @@
 namespace frt {
 namespace {
 
-constexpr int kThreads = 224;
+constexpr int kThreads = 256;
+// Named barrier of the issuer / observer hand-off (warps 1 and 7); id 1 serves the
+// epilogue warps, id 0 is __syncthreads.
+constexpr int kBarHandoff = 4;
 constexpr int kBM = 128;         // output pixels per tile: 16 rows x 8 columns
 constexpr int kTileW = 8;        // one 8-row operand group = one tile row
 constexpr int kTileH = 16;
@@ -284,8 +290,19 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
                     mbar_wait_drain(smem_u32(&bars.b_full[i % p.b_stages]), (i / p.b_stages) & 1, lim);
         }
     } else if (warp == 1) {
-        // ======================= MMA issuer (one thread of the leader) =======================
-        if (lane == 0 && leader) {
+        // ============ MMA issuer (a converged warp of the leader; lane 0 issues) ============
+        // The warp never touches an mbarrier in its loops: the observer warp (warp 7) waits
+        // for every barrier the next MMAs need and meets it at the hand-off named barrier.
+        // (A shared-memory access by the issuing thread behind queued MMAs waits behind
+        // their operand reads, ~400 cycles per weight stage measured; a named barrier reads
+        // no shared memory.) Both warps pass the same barriers in the same order whatever
+        // happens, so neither can strand the other.
+        if (leader) {
+            const uint32_t lead = lane == 0 ? 1u : 0u;
+            auto handoff = [&]() {
+                named_bar_sync(kBarHandoff, 64);
+                tc_fence_after();
+            };
             // descriptors are linear in the 16-byte start address (addresses stay below
             // 256 KB, so the 14-bit field never carries): tap (dh, dw) of halo stage sa
             // is da0 + sa * a_step + dh * halo_w * 8 + dw, k-step k adds 2 k
@@ -295,78 +312,86 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
             const uint32_t row_skip = uint32_t((p.halo_w - p.kw) * 8);
             const uint32_t b_step = uint32_t(p.b_stage >> 4);
             int sa = 0, sb = 0;
-            uint32_t pa = 0, pb = 0;
-            int ia = 0, ib = 0;
             int tl = 0;
-            bool ok = true;
-            for (int t = c_first; t < p.n_tiles && ok; t += c_stride, ++tl) {
+            for (int t = c_first; t < p.n_tiles; t += c_stride, ++tl) {
                 const int b = tl & 1;
-                if (tl >= 2 &&
-                    !mbar_wait(smem_u32(&bars.acc_empty[b]), ((tl >> 1) - 1) & 1, lim, abort)) {
-                    report(p.status, abort, 1, -1 - tl);
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
+                if (tl >= 2) handoff();                      // accumulator b drained
                 const uint32_t d = tmem + uint32_t(b * BN);
                 uint32_t accumulate = 0;
-                for (int hi = 0; hi < nhalo && ok; ++hi, ++ia) {
-                    if (!mbar_test_wait(smem_u32(&bars.a_full[sa]), pa) &&
-                        !mbar_wait(smem_u32(&bars.a_full[sa]), pa, lim, abort)) {
-                        report(p.status, abort, 1, ia);
-                        ok = false;
-                        break;
-                    }
+                for (int hi = 0; hi < nhalo; ++hi) {
+                    handoff();                               // halo stage sa landed
                     uint64_t da = da0 + uint64_t(uint32_t(sa) * a_step);
-                    // a weight stage holds tb consecutive taps of one kernel row: one wait
-                    // per tb * 4 MMAs (a wait issued behind MMAs costs the issuing thread
-                    // ~200 cycles, which only a long enough MMA queue hides)
-                    for (int dh = 0; dh < p.kh && ok; ++dh, da += row_skip) {
-                        for (int dw = 0; dw < p.kw; dw += p.tb, ++ib) {
-                            if (!mbar_test_wait(smem_u32(&bars.b_full[sb]), pb) &&
-                                !mbar_wait(smem_u32(&bars.b_full[sb]), pb, lim, abort)) {
-                                report(p.status, abort, 4, ib);
-                                ok = false;
-                                break;
-                            }
-                            tc_fence_after();
+                    // a weight stage holds tb consecutive taps of one kernel row: one
+                    // hand-off per tb * 4 MMAs
+                    for (int dh = 0; dh < p.kh; ++dh, da += row_skip) {
+                        for (int dw = 0; dw < p.kw; dw += p.tb) {
+                            handoff();                       // weight stage sb landed
                             uint64_t db = db0 + uint64_t(uint32_t(sb) * b_step);
                             for (int u = 0; u < p.tb; ++u, da += 8, db += uint64_t(C::B_BYTES >> 4)) {
 #pragma unroll
                                 for (int k = 0; k < kBK / 16; ++k) {
                                     if (PAIR)
-                                        umma_ss_pair(d, da + uint64_t(2 * k), db + uint64_t(2 * k),
-                                                     C::IDESC, accumulate);
+                                        umma_ss_pair_if(lead, d, da + uint64_t(2 * k),
+                                                        db + uint64_t(2 * k), C::IDESC, accumulate);
                                     else
-                                        umma_ss(d, da + uint64_t(2 * k), db + uint64_t(2 * k), C::IDESC,
-                                                accumulate);
+                                        umma_ss_if(lead, d, da + uint64_t(2 * k), db + uint64_t(2 * k),
+                                                   C::IDESC, accumulate);
                                     accumulate = 1;
                                 }
                             }
-                            if (PAIR) umma_commit_pair(smem_u32(&bars.b_empty[sb]), 0x3);
-                            else umma_commit(smem_u32(&bars.b_empty[sb]));
+                            if (PAIR) umma_commit_pair_if(lead, smem_u32(&bars.b_empty[sb]), 0x3);
+                            else umma_commit_if(lead, smem_u32(&bars.b_empty[sb]));
+                            if (++sb == p.b_stages) sb = 0;
+                        }
+                    }
+                    if (PAIR) umma_commit_pair_if(lead, smem_u32(&bars.a_empty[sa]), 0x3);
+                    else umma_commit_if(lead, smem_u32(&bars.a_empty[sa]));
+                    if (++sa == p.a_stages) sa = 0;
+                }
+                if (PAIR) umma_commit_pair_if(lead, smem_u32(&bars.acc_full[b]), 0x3);
+                else umma_commit_if(lead, smem_u32(&bars.acc_full[b]));
+            }
+            if (PAIR) umma_commit_pair_if(lead, smem_u32(&bars.drain), 0x1);
+            else umma_commit_if(lead, smem_u32(&bars.drain));
+            mbar_wait_drain(smem_u32(&bars.drain), 0, lim);
+        }
+    } else if (warp == 7) {
+        // ======== observer (leader): waits for what the issuer's next MMAs need ========
+        // After a wait gives up (or another role raised the abort flag) the remaining
+        // hand-offs pass without waiting; the issuer then finishes on stale operands, which
+        // the recorded error status marks as void.
+        if (leader) {
+            bool ok = true;
+            auto observe = [&](uint32_t bar, uint32_t parity, int role, int where) {
+                if (ok) {
+                    ok = __all_sync(0xffffffffu, mbar_wait(bar, parity, lim, abort));
+                    if (!ok && lane == 0) report(p.status, abort, role, where);
+                }
+                named_bar_sync(kBarHandoff, 64);
+            };
+            int sa = 0, sb = 0;
+            uint32_t pa = 0, pb = 0;
+            int ia = 0, ib = 0;
+            int tl = 0;
+            for (int t = c_first; t < p.n_tiles; t += c_stride, ++tl) {
+                const int b = tl & 1;
+                if (tl >= 2) observe(smem_u32(&bars.acc_empty[b]), ((tl >> 1) - 1) & 1, 1, -1 - tl);
+                for (int hi = 0; hi < nhalo; ++hi, ++ia) {
+                    observe(smem_u32(&bars.a_full[sa]), pa, 1, ia);
+                    for (int dh = 0; dh < p.kh; ++dh)
+                        for (int dw = 0; dw < p.kw; dw += p.tb, ++ib) {
+                            observe(smem_u32(&bars.b_full[sb]), pb, 4, ib);
                             if (++sb == p.b_stages) {
                                 sb = 0;
                                 pb ^= 1;
                             }
                         }
-                    }
-                    if (!ok) break;
-                    if (PAIR) umma_commit_pair(smem_u32(&bars.a_empty[sa]), 0x3);
-                    else umma_commit(smem_u32(&bars.a_empty[sa]));
                     if (++sa == p.a_stages) {
                         sa = 0;
                         pa ^= 1;
                     }
                 }
-                if (ok) {
-                    if (PAIR) umma_commit_pair(smem_u32(&bars.acc_full[b]), 0x3);
-                    else umma_commit(smem_u32(&bars.acc_full[b]));
-                }
             }
-            if (PAIR) umma_commit_pair(smem_u32(&bars.drain), 0x1);
-            else umma_commit(smem_u32(&bars.drain));
-            mbar_wait_drain(smem_u32(&bars.drain), 0, lim);
         }
     } else {
         // ====================================== epilogue =====================================

@@ -2,15 +2,17 @@
 // fp32 accumulation in TMEM, for the linear projections around the chunk attention of a
 // DiT block (QKV projection in front of it, output projection after it).
 //
-// Persistent kernel, one CTA per SM, 320 threads:
+// Persistent kernel, one CTA per SM, 352 threads:
 //   warp 0      TMA producer: two k-blocks of A (128 x 64 each) and of B (BN x 64 each)
 //               per ring stage, 128-byte swizzle, through a shared-memory ring (with K a
 //               multiple of 64, one box per operand loads both k-blocks through a 3D view
 //               (64, rows, K / 64) of the matrix);
-//   warp 1      TMEM allocator + single-thread tcgen05.mma issuer (M = 128, N = BN, K = 16
-//               per instruction, eight per stage: one barrier wait per eight MMAs, since a
-//               shared-memory access by the issuing thread behind queued MMAs stalls it
-//               ~140 cycles);
+//   warp 1      TMEM allocator + tcgen05.mma issuer (M = 128, N = BN, K = 16 per
+//               instruction, eight per stage): a converged warp whose lane 0 issues; it
+//               touches no mbarrier in its loop (a shared-memory access by the issuing
+//               thread behind queued MMAs stalls it behind their operand reads);
+//   warp 10     observer: waits on the stage and accumulator barriers in the issuer's
+//               order and hands each off to it through a named barrier;
 //   warps 2-9   epilogue: two warps per TMEM lane quarter, each thread one accumulator
 //               row (TMEM lane) and one half of every column unit: each 128-byte
 //               column unit of the tile (32 fp32 or 64 bf16 columns) is staged in a 128-byte-swizzled shared-memory slab and written
@@ -46,8 +48,11 @@ namespace frt {
 
 namespace {
 
-constexpr int kThreads = 320;
+constexpr int kThreads = 352;
 constexpr int kEpiThreads = 256;   // warps 2-9
+// Named barrier of the issuer / observer hand-off (warps 1 and 10); id 1 serves the
+// epilogue warps, id 0 is __syncthreads.
+constexpr int kBarHandoff = 4;
 constexpr int kBM = 128;
 constexpr int kBK = 64;          // one 128-byte swizzle atom of bf16
 constexpr int kMaxStages = 6;
@@ -208,34 +213,32 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
                     mbar_wait_drain(smem_u32(&bars.full[i % kStages]), (i / kStages) & 1, lim);
         }
     } else if (warp == 1) {
-        // ======================= MMA issuer (one thread of the leader) =======================
-        if (lane == 0 && leader) {
+        // ============ MMA issuer (a converged warp of the leader; lane 0 issues) ============
+        // The warp never touches an mbarrier in its loop: the observer warp (warp 10) waits
+        // for every barrier the next MMAs need and meets it at the hand-off named barrier.
+        // (A shared-memory access by the issuing thread behind queued MMAs waits behind
+        // their operand reads, ~300 cycles per stage measured; a named barrier reads no
+        // shared memory.) Both warps pass the same barriers in the same order whatever
+        // happens, so neither can strand the other.
+        if (leader) {
+            const uint32_t lead = lane == 0 ? 1u : 0u;
+            auto handoff = [&]() {
+                named_bar_sync(kBarHandoff, 64);
+                tc_fence_after();
+            };
             // descriptors are linear in the 16-byte start address: a K step of 16 bf16
             // inside the 128-byte swizzle atom adds 32 bytes (2 units)
             const uint64_t da0 = sdesc_sw128(sbase, 16, 1024);
             const uint64_t db0 = sdesc_sw128(sbase + kKPS * C::A_BYTES, 16, 1024);
             int it = 0;
             int tl = 0;
-            bool ok = true;
-            for (int t = c_first; t < n_tiles && ok; t += c_stride, ++tl) {
+            for (int t = c_first; t < n_tiles; t += c_stride, ++tl) {
                 const int b = tl & 1;
-                if (tl >= 2 &&
-                    !mbar_wait(smem_u32(&bars.acc_empty[b]), ((tl >> 1) - 1) & 1, lim, abort)) {
-                    report(p.status, abort, 1, -1 - tl);
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
+                if (tl >= 2) handoff();                      // accumulator b drained
                 const uint32_t d = tmem + uint32_t(b * BN);
                 for (int kb = 0; kb < nk; kb += kKPS, ++it) {
                     const int s = it % kStages;
-                    if (!mbar_test_wait(smem_u32(&bars.full[s]), (it / kStages) & 1) &&
-                        !mbar_wait(smem_u32(&bars.full[s]), (it / kStages) & 1, lim, abort)) {
-                        report(p.status, abort, 1, it);
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
+                    handoff();                               // stage s landed
                     const uint64_t so = uint64_t((s * C::STAGE) >> 4);
 #pragma unroll
                     for (int h = 0; h < kKPS; ++h) {
@@ -246,23 +249,46 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
                         for (int k = 0; k < kBK / 16; ++k) {
                             const uint32_t acc = (kb + h > 0 || k > 0) ? 1u : 0u;
                             if (PAIR)
-                                umma_ss_pair(d, da + uint64_t(2 * k), db + uint64_t(2 * k), C::IDESC, acc);
+                                umma_ss_pair_if(lead, d, da + uint64_t(2 * k), db + uint64_t(2 * k),
+                                                C::IDESC, acc);
                             else
-                                umma_ss(d, da + uint64_t(2 * k), db + uint64_t(2 * k), C::IDESC, acc);
+                                umma_ss_if(lead, d, da + uint64_t(2 * k), db + uint64_t(2 * k),
+                                           C::IDESC, acc);
                         }
                     }
-                    if (PAIR) umma_commit_pair(smem_u32(&bars.empty[s]), 0x3);
-                    else umma_commit(smem_u32(&bars.empty[s]));
+                    if (PAIR) umma_commit_pair_if(lead, smem_u32(&bars.empty[s]), 0x3);
+                    else umma_commit_if(lead, smem_u32(&bars.empty[s]));
                 }
-                if (ok) {
-                    if (PAIR) umma_commit_pair(smem_u32(&bars.acc_full[b]), 0x3);
-                    else umma_commit(smem_u32(&bars.acc_full[b]));
-                }
+                if (PAIR) umma_commit_pair_if(lead, smem_u32(&bars.acc_full[b]), 0x3);
+                else umma_commit_if(lead, smem_u32(&bars.acc_full[b]));
             }
             // drain: all issued MMAs complete before TMEM is released
-            if (PAIR) umma_commit_pair(smem_u32(&bars.drain), 0x1);
-            else umma_commit(smem_u32(&bars.drain));
+            if (PAIR) umma_commit_pair_if(lead, smem_u32(&bars.drain), 0x1);
+            else umma_commit_if(lead, smem_u32(&bars.drain));
             mbar_wait_drain(smem_u32(&bars.drain), 0, lim);
+        }
+    } else if (warp == 10) {
+        // ======== observer (leader): waits for what the issuer's next MMAs need ========
+        // After a wait gives up (or another role raised the abort flag) the remaining
+        // hand-offs pass without waiting; the issuer then finishes on stale operands, which
+        // the recorded error status marks as void.
+        if (leader) {
+            bool ok = true;
+            auto observe = [&](uint32_t bar, uint32_t parity, int where) {
+                if (ok) {
+                    ok = __all_sync(0xffffffffu, mbar_wait(bar, parity, lim, abort));
+                    if (!ok && lane == 0) report(p.status, abort, 1, where);
+                }
+                named_bar_sync(kBarHandoff, 64);
+            };
+            int it = 0;
+            int tl = 0;
+            for (int t = c_first; t < n_tiles; t += c_stride, ++tl) {
+                const int b = tl & 1;
+                if (tl >= 2) observe(smem_u32(&bars.acc_empty[b]), ((tl >> 1) - 1) & 1, -1 - tl);
+                for (int kb = 0; kb < nk; kb += kKPS, ++it)
+                    observe(smem_u32(&bars.full[it % kStages]), (it / kStages) & 1, it);
+            }
         }
     } else {
         // ====================================== epilogue =====================================
