@@ -33,6 +33,14 @@ int frt_selftest_umma_tile(const void* a, const void* b, float* c, int b_mn_majo
 int frt_selftest_umma_pair(const void* a, const void* b, float* c, unsigned* taddrs,
                            int* dev_status, void* cuda_stream);
 
+/* The P.V form of the same pair MMA: A (device [256, 128] bf16, row-major) is staged in
+ * TMEM (CTA r its rows [128 r, 128 r + 128), packed bf16 pairs) and used as the TMEM
+ * operand; b is device [128, 128] bf16 row-major read as the MN-major B (K rows x N
+ * columns), CTA r holding N columns [64 r, 64 r + 64). c = A . b, device [256, 128] fp32.
+ * Returns 0 on launch success, < 0 on an argument/launch error. */
+int frt_selftest_umma_pair_pv(const void* a, const void* b, float* c, unsigned* taddrs,
+                              int* dev_status, void* cuda_stream);
+
 /* Force the output-column tile width of every later projection launch (frt_gemm_bf16,
  * frt_block_step, frt_gemm_plan) to bn in {128, 192, 256}; 0 restores the automatic
  * choice. Process-wide and not thread-safe: for tests that cover every width. Returns

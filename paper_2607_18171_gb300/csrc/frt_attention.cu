@@ -568,7 +568,21 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 bulk_wait_read<0>();
             }
         };
-        if (n_parts == 1) {
+        // the item's split coordinates, re-derived from the block index here instead of
+        // kept live through the KV loop (registers are scarce in the softmax warps: kept
+        // live, they made the compiler spill inside the fused RoPE variant)
+        int e_split = 0, e_parts = 1, e_tail = 0;
+        {
+            int cid;
+            asm volatile("mov.u32 %0, %%ctaid.x;" : "=r"(cid));
+            if (cid >= p.n_full) {
+                const int v = cid - p.n_full;
+                e_tail = v / p.n_split;
+                e_split = v - e_tail * p.n_split;
+                e_parts = p.n_split;
+            }
+        }
+        if (e_parts == 1) {
             if (ok) {
                 // O / l -> out
                 tc_fence_after();
@@ -587,8 +601,8 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             }
             store_out();
         } else {
-            // unnormalised partial of this split -> scratch (rows of tile (tail, split, g))
-            const int prow_tile = int((size_t(tail) * n_parts + split) * 2 * kBM) + g * kBM;
+            // unnormalised partial of this split -> scratch (rows of tile (tail group, split, g))
+            const int prow_tile = int((size_t(e_tail) * e_parts + e_split) * 2 * kBM) + g * kBM;
             if (ok) {
                 tc_fence_after();
 #pragma unroll 1
@@ -616,21 +630,21 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             // the last split of this query group to finish merges all partials
             named_bar_sync(1, 256);
             if (threadIdx.x == 128) {
-                const int old = atomicAdd(p.counters + tail, 1);
-                const int last = (old == n_parts - 1);
-                if (last) p.counters[tail] = 0;    // every split has counted: reset for reuse
+                const int old = atomicAdd(p.counters + e_tail, 1);
+                const int last = (old == e_parts - 1);
+                if (last) p.counters[e_tail] = 0;    // every split has counted: reset for reuse
                 bars->last_split = last;
             }
             named_bar_sync(1, 256);
             if (bars->last_split) {
                 __threadfence();
                 fence_proxy_async_global();
-                const int prow0 = int(size_t(tail) * n_parts * 2 * kBM) + g * kBM;
+                const int prow0 = int(size_t(e_tail) * e_parts * 2 * kBM) + g * kBM;
                 float2 ml[kMaxSplit];
 #pragma unroll
                 for (int r = 0; r < kMaxSplit; ++r)
-                    ml[r] = (r == split) ? make_float2(m_run, l_run)
-                            : (r < n_parts) ? __ldcg(&p.part_ml[prow0 + r * 2 * kBM + row])
+                    ml[r] = (r == e_split) ? make_float2(m_run, l_run)
+                            : (r < e_parts) ? __ldcg(&p.part_ml[prow0 + r * 2 * kBM + row])
                                               : make_float2(-INFINITY, 0.0f);
                 float mref = -INFINITY;
 #pragma unroll
@@ -639,7 +653,7 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 float lsum = 0.0f;
 #pragma unroll
                 for (int r = 0; r < kMaxSplit; ++r) {
-                    wr[r] = (r < n_parts) ? ex2_approx(ml[r].x - mref) : 0.0f;
+                    wr[r] = (r < e_parts) ? ex2_approx(ml[r].x - mref) : 0.0f;
                     lsum += wr[r] * ml[r].y;
                 }
                 const float w_own = ex2_approx(m_run - mref);
@@ -652,8 +666,8 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
                 int phase = 0;
 #pragma unroll
                 for (int r = 0; r < kMaxSplit; ++r) {
-                    if (r >= n_parts) continue;
-                    const bool own = (r == split);
+                    if (r >= e_parts) continue;
+                    const bool own = (r == e_split);
                     if (!own) {
                         const uint32_t fb = smem_u32(&bars->epi_full[g]);
                         if (ok && leader) {

@@ -132,9 +132,13 @@ constexpr int kPairA = 128 * 128 * 2;
 constexpr int kPairB = 64 * 128 * 2;
 constexpr int kPairSmem = kPairA + kPairB + 1024;
 
+// pv = 1: the P.V form of the attention's pair MMA instead: A (256 x 128, K-major) is
+// staged in TMEM (CTA r its 128 rows, packed bf16 pairs in columns [128, 192)) and B is
+// the [128 (K), 128 (N)] row-major matrix read MN-major, CTA r holding the N columns
+// [64 r, 64 r + 64): C = A B.
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(128, 1)
 umma_pair_kernel(const __grid_constant__ CUtensorMap a_map, const __grid_constant__ CUtensorMap b_map,
-                 float* c, uint32_t* taddrs, int* status) {
+                 float* c, uint32_t* taddrs, int* status, int pv) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
@@ -163,22 +167,58 @@ umma_pair_kernel(const __grid_constant__ CUtensorMap a_map, const __grid_constan
     if (threadIdx.x == 0) {
         const uint32_t full_leader = mapa_shared(smem_u32(&full), 0);
         if (rank == 0) mbar_arrive_expect_tx(smem_u32(&full), 2 * (kPairA + kPairB));
-        for (int cb = 0; cb < 2; ++cb) {
+        for (int cb = 0; cb < 2; ++cb)
             tma_load_2d_pair(sA + cb * (128 * 128), &a_map, full_leader, cb * 64, int(rank) * 128);
-            tma_load_2d_pair(sB + cb * (64 * 128), &b_map, full_leader, cb * 64, int(rank) * 64);
+        if (pv)   // this CTA's 64 N columns of all 128 K rows: one 128-byte-wide box
+            tma_load_2d_pair(sB, &b_map, full_leader, int(rank) * 64, 0);
+        else
+            for (int cb = 0; cb < 2; ++cb)
+                tma_load_2d_pair(sB + cb * (64 * 128), &b_map, full_leader, cb * 64, int(rank) * 64);
+    }
+    // every CTA waits for the pair's loads (they complete on the leader's barrier), then
+    // in the P.V form stages its A rows in TMEM
+    bool got = true;
+    if (pv) {
+        if (rank == 0) got = mbar_wait(smem_u32(&full), 0, lim, &abort_flag);
+        cluster_sync_all();   // the leader has seen every byte of both CTAs land
+        got = __all_sync(0xffffffffu, got);
+        const int row = threadIdx.x;
+        uint32_t regs[64];
+        for (int ch = 0; ch < 16; ++ch) {
+            const int cb = ch >> 3, cc = ch & 7;
+            const uint4 v = *reinterpret_cast<const uint4*>(smem + cb * (128 * 128) + row * 128 +
+                                                            ((cc ^ (row & 7)) << 4));
+            regs[4 * ch + 0] = v.x; regs[4 * ch + 1] = v.y;
+            regs[4 * ch + 2] = v.z; regs[4 * ch + 3] = v.w;
         }
-        if (rank == 0) {
-            if (mbar_wait(smem_u32(&full), 0, lim, &abort_flag)) {
-                tc_fence_after();
-                const uint32_t idesc = idesc_bf16_f32(256, 128, false);
-                for (int k = 0; k < 8; ++k) {
+        const uint32_t lane_off = uint32_t(warp * 32) << 16;
+        uint32_t r32[32];
+        for (int h = 0; h < 2; ++h) {
+            for (int i = 0; i < 32; ++i) r32[i] = regs[32 * h + i];
+            tmem_st32(tmem + lane_off + 128 + 32 * h, r32);
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        cluster_sync_all();   // both CTAs' A rows are in TMEM
+        tc_fence_after();
+    }
+    if (threadIdx.x == 0 && rank == 0) {
+        if (!pv) got = mbar_wait(smem_u32(&full), 0, lim, &abort_flag);
+        if (got) {
+            tc_fence_after();
+            const uint32_t idesc = idesc_bf16_f32(256, 128, pv != 0);
+            for (int k = 0; k < 8; ++k) {
+                if (pv) {
+                    umma_ts_pair(tmem, tmem + 128 + k * 8, sdesc_sw128(sB + k * (16 * 128), 16384, 1024),
+                                 idesc, k > 0);
+                } else {
                     const uint32_t aoff = (k >> 2) * (128 * 128) + (k & 3) * 32;
                     const uint32_t boff = (k >> 2) * (64 * 128) + (k & 3) * 32;
                     umma_ss_pair(tmem, sdesc_sw128(sA + aoff, 16, 1024),
                                  sdesc_sw128(sB + boff, 16, 1024), idesc, k > 0);
                 }
-                umma_commit_pair(smem_u32(&done), 0x3);
             }
+            umma_commit_pair(smem_u32(&done), 0x3);
         }
     }
     bool ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&done), 0, lim, &abort_flag));
@@ -297,7 +337,20 @@ extern "C" int frt_selftest_umma_pair(const void* a, const void* b, float* c, un
                              kPairSmem) != cudaSuccess)
         return -3;
     umma_pair_kernel<<<2, 128, kPairSmem, static_cast<cudaStream_t>(cuda_stream)>>>(
-        am, bm, c, taddrs, dev_status);
+        am, bm, c, taddrs, dev_status, 0);
+    return cudaGetLastError() == cudaSuccess ? 0 : -4;
+}
+
+extern "C" int frt_selftest_umma_pair_pv(const void* a, const void* b, float* c, unsigned* taddrs,
+                                         int* dev_status, void* cuda_stream) {
+    if (!a || !b || !c || !taddrs || !dev_status) return -1;
+    CUtensorMap am, bm;
+    if (map_2d(&am, a, 256, 128) || map_2d(&bm, b, 128, 128)) return -2;
+    if (cudaFuncSetAttribute(umma_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             kPairSmem + kPairB) != cudaSuccess)
+        return -3;
+    umma_pair_kernel<<<2, 128, kPairSmem + kPairB, static_cast<cudaStream_t>(cuda_stream)>>>(
+        am, bm, c, taddrs, dev_status, 1);
     return cudaGetLastError() == cudaSuccess ? 0 : -4;
 }
 

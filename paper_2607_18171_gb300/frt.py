@@ -98,6 +98,7 @@ def lib() -> ctypes.CDLL:
         "frt_selftest_umma_tile": (I, [P, P, P, I, I, I, I, P, P]),
         "frt_selftest_wait_timeout": (I, [P, LL, P]),
         "frt_selftest_umma_pair": (I, [P, P, P, P, P, P]),
+        "frt_selftest_umma_pair_pv": (I, [P, P, P, P, P, P]),
         "frt_selftest_gemm_force_bn": (I, [I]),
         "frt_steps_create": (P, [I, I, I, I, I, I]),
         "frt_steps_configure": (I, [P, ctypes.POINTER(Config)]),
@@ -526,13 +527,15 @@ def selftest_umma_tile(a: torch.Tensor, b: torch.Tensor, b_mn_major: bool, lbo: 
     return c
 
 
-def selftest_umma_pair(a: torch.Tensor, b: torch.Tensor):
-    """(C [256,128] fp32, TMEM addresses the two CTAs got) for C = A B^T on a CTA pair."""
+def selftest_umma_pair(a: torch.Tensor, b: torch.Tensor, pv: bool = False):
+    """(C [256,128] fp32, TMEM addresses the two CTAs got) for C = A B^T on a CTA pair, or
+    with pv=True C = A B with A staged in TMEM and B read MN-major (the P.V form)."""
     c = torch.empty(256, 128, dtype=torch.float32, device="cuda")
     taddrs = torch.zeros(2, dtype=torch.int32, device="cuda")
     status = torch.zeros(1, dtype=torch.int32, device="cuda")
-    rc = lib().frt_selftest_umma_pair(_ptr(a), _ptr(b), _ptr(c), _ptr(taddrs), _ptr(status),
-                                      ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+    fn = lib().frt_selftest_umma_pair_pv if pv else lib().frt_selftest_umma_pair
+    rc = fn(_ptr(a), _ptr(b), _ptr(c), _ptr(taddrs), _ptr(status),
+            ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
     if rc != 0:
         raise FrtError(4, f"pair selftest launch failed ({rc})")
     torch.cuda.synchronize()

@@ -75,3 +75,14 @@ def test_umma_cta_pair_tile(frt):
     c, taddrs = frt.selftest_umma_pair(a.cuda(), b.cuda())
     assert taddrs[0] == taddrs[1]      # one allocation shared by the pair
     _check(c, a.double() @ b.double().T)
+
+
+def test_umma_cta_pair_pv_tile(frt):
+    """The attention's P.V product on a CTA pair: A (P) from TMEM, B (V) MN-major and
+    split by its N columns (head_dim halves) across the two CTAs."""
+    g = torch.Generator().manual_seed(5)
+    a = torch.randn(256, 128, generator=g).to(torch.bfloat16)
+    b = torch.randn(128, 128, generator=g).to(torch.bfloat16)
+    c, taddrs = frt.selftest_umma_pair(a.cuda(), b.cuda(), pv=True)
+    assert taddrs[0] == taddrs[1]
+    _check(c, a.double() @ b.double())
