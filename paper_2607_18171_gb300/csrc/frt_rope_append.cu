@@ -34,6 +34,7 @@ struct StagedParams {
     int vec_per_head_log2;   // log2(head_dim / 8)
     int tok_per_block;       // tokens per stage
     int stages;              // ring depth (<= kMaxStages)
+    int coop;                // rotation: all worker warps share each token (wide rows)
     const uint8_t* a_lo;     // destination extents [lo, hi) checked by the FRT_DEBUG build
     const uint8_t* a_hi;
     const uint8_t* b_lo;
@@ -133,11 +134,15 @@ __global__ void __launch_bounds__(kThreads, 1) staged_rows_kernel(const __grid_c
             bulk_wait_read<0>();
         }
     } else {
-        // one warp per token: a lane's 16-byte vectors all sit at the same head_dim
-        // offset (32 is a multiple of the vectors per head), so its four (cos, sin)
-        // pairs are fetched once per token and reused for every head
+        // Narrow rows: one warp per token. Wide rows (p.coop): all seven warps share each
+        // token, so a stage of one or two wide tokens does not leave five warps idle. In
+        // both a lane's 16-byte vectors all sit at the same head_dim offset (the stride,
+        // 32 or 224 vectors, is a multiple of the vectors per head), so its four
+        // (cos, sin) pairs are fetched once per token and reused for every head.
         const int wid = warp - 1;
         const int d0 = (lane & ((1 << p.vec_per_head_log2) - 1)) * 8;
+        const int t_first = p.coop ? 0 : wid, t_step = p.coop ? 1 : kWorkers / 32;
+        const int v_first = p.coop ? wid * 32 + lane : lane, v_step = p.coop ? kWorkers : 32;
         for (int i = 0; i < my_n; ++i) {
             const int s = i % kStages;
             if (!mbar_wait(smem_u32(&full[s]), (i / kStages) & 1, lim, abort)) {
@@ -149,7 +154,7 @@ __global__ void __launch_bounds__(kThreads, 1) staged_rows_kernel(const __grid_c
             for (int ab = 0; ab < 2; ++ab) {
                 if (!(ab == 0 ? p.rot_a : p.rot_b)) continue;
                 uint4* rows = reinterpret_cast<uint4*>(ring + s * 2 * half + ab * half);
-                for (int t = wid; t < nt; t += kWorkers / 32) {
+                for (int t = t_first; t < nt; t += t_step) {
                     const int tok = tok0 + t;
                     const int f = tok / p.ra.tpf;
                     const int rem = tok - f * p.ra.tpf;
@@ -159,7 +164,7 @@ __global__ void __launch_bounds__(kThreads, 1) staged_rows_kernel(const __grid_c
 #pragma unroll
                     for (int q = 0; q < 4; ++q) cs[q] = rope_cs(p.ra, s_t, (d0 >> 1) + q, f, r, col);
                     uint4* tr = rows + size_t(t) * p.vec_per_tok;
-                    for (int v = lane; v < p.vec_per_tok; v += 32) {
+                    for (int v = v_first; v < p.vec_per_tok; v += v_step) {
                         uint4 x = tr[v];
                         x.x = rope_pair(x.x, cs[0].x, cs[0].y);
                         x.y = rope_pair(x.y, cs[1].x, cs[1].y);
@@ -180,6 +185,11 @@ cudaError_t launch_staged(StagedParams& sp, cudaStream_t st) {
     sp.tok_per_block = std::max(1, std::min(sp.n_tok, kStageTarget / (2 * sp.row_bytes)));
     const int stage_bytes = 2 * sp.tok_per_block * sp.row_bytes;
     sp.stages = std::min(kMaxStages, kSmemBudget / stage_bytes);
+    // rows of at least two vectors per worker thread are rotated by all worker warps
+    // together (measured at 40 heads x 128, 10 KB rows, two tokens per stage: 720p append
+    // 5547 -> 6053 GB/s); narrower rows keep one warp per token (3 KB rows measured
+    // 3410 -> 2112 GB/s the other way)
+    sp.coop = sp.vec_per_tok >= 2 * kWorkers ? 1 : 0;
     if (sp.stages < 2) return cudaErrorInvalidValue;   // rows too large (create() prevents it)
     sp.wait_limit_ns = 2000000000ull;
     const int smem = sp.stages * stage_bytes;
