@@ -14,9 +14,10 @@
 //                 S_g  = Q_g K_j^T  A, B from shared memory (K-major, 128-byte swizzle)
 //                 O_g += P_g V_j    A = P from TMEM, B = V from shared memory (MN-major)
 //               issued as PV_0(j), S_0(j+1), PV_1(j), S_1(j+1): the tiles alternate
-//   warp 2      observer: waits on the K/V and P barriers the issuer needs next and hands
-//               off to it through a named barrier (the issuer touches no mbarrier in the
-//               KV loop)
+//   warp 2      observer: waits on the K/V barriers the issuer needs next and hands
+//               off to it through a named barrier; the softmax groups meet the issuer at
+//               their own named barriers when P is in TMEM (the issuer touches no mbarrier
+//               in the KV loop)
 //   warp 3      idle
 //   warps 4-7   softmax group 0 (query tile 0), one thread per query row
 //   warps 8-11  softmax group 1 (query tile 1)
@@ -51,9 +52,11 @@ constexpr int kBM = 128;   // query rows per tile
 constexpr int kBN = 128;   // KV rows per tile
 constexpr float kOverflowGuard = 1.152921504606846976e18f;   // 2^60
 constexpr int kTimeoutCode = 6;  // FRT_ERR_TIMEOUT
-// Named barrier of the issuer / observer hand-off (warps 1 and 2). Ids 1-3 serve the
-// softmax groups' epilogues, id 0 is __syncthreads.
+// Named barriers: 0 __syncthreads, 1-3 the softmax groups' epilogues, 4 the issuer /
+// observer hand-off (warps 1 and 2), 5 and 6 P_0 and P_1 ready (softmax group g's 128
+// threads and the issuer warp's 32).
 constexpr int kBarHandoff = 4;
+constexpr int kBarP = 5;
 
 template <int D>
 struct Cfg {
@@ -73,7 +76,6 @@ struct Bars {
     uint64_t q_full;
     uint64_t q_ready[2];
     uint64_t s_full[2];
-    uint64_t p_full[2];
     uint64_t o_done[2];
     uint64_t drain[2];
     uint64_t kv_full[8];
@@ -166,7 +168,6 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
         for (int g = 0; g < 2; ++g) {
             mbar_init(smem_u32(&bars->q_ready[g]), kBM);
             mbar_init(smem_u32(&bars->s_full[g]), 1);
-            mbar_init(smem_u32(&bars->p_full[g]), kBM);
             mbar_init(smem_u32(&bars->o_done[g]), 1);
         }
         mbar_init(smem_u32(&bars->drain[0]), 1);
@@ -279,6 +280,11 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             named_bar_sync(kBarHandoff, 64);
             tc_fence_after();
         };
+        // P_g(j) written to TMEM by softmax group g (its 128 threads arrive)
+        auto take_p = [&](int g) {
+            named_bar_sync(kBarP + g, 160);
+            tc_fence_after();
+        };
         // MMA groups: S_g = Q_g K^T (8 MMAs over D) and O_g += P_g V (8 MMAs over the KV
         // tile). `mid(k)` runs after MMA k of a group, in the shadow of the running MMA.
         auto issue_s = [&](int g, int stage, auto&& mid) {
@@ -305,8 +311,8 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             }
         };
         auto nop = [](int) {};
-        // Hand-off sequence (the observer follows the same one): K_0/V_0; then per KV step
-        // j: P_0(j), K_{j+1}/V_{j+1} (if any), P_1(j) (two tiles).
+        // Hand-off sequence (the observer follows the same one): K_0/V_0, then per KV step
+        // j the pair K_{j+1}/V_{j+1} (if any); P_g(j) comes straight from group g.
         handoff();
         issue_s(0, 0, nop);
         if (ng == 2) issue_s(1, 0, nop);
@@ -314,7 +320,7 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
         int sv = 1 % C::STAGES, sk = 2 % C::STAGES;   // ring slots of V_j and K_{j+1}
         for (int j = 0; j < n_tiles; ++j) {
             const bool more = (j + 1) < n_tiles;
-            handoff();                                  // P_0(j)
+            take_p(0);                                  // P_0(j)
             // the release of step j-1 rides in the shadow of PV_0(j)'s second MMA
             issue_o(0, sv, j > 0, [&](int k) {
                 if (k == 0 && more) handoff();          // K_{j+1}, V_{j+1}
@@ -323,7 +329,7 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             if (more) issue_s(0, sk, nop);
             else umma_commit_if(iss, smem_u32(&bars->o_done[0]));
             if (ng == 2) {
-                handoff();                              // P_1(j)
+                take_p(1);                              // P_1(j)
                 issue_o(1, sv, j > 0, nop);
                 if (more) issue_s(1, sk, nop);
                 else umma_commit_if(iss, smem_u32(&bars->o_done[1]));
@@ -352,11 +358,8 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
         // warp saw pair j, so the parity of kv_full[j % 4] is never ambiguous.
         auto kv_bar = [&](int jj) { return smem_u32(&bars->kv_full[jj & 3]); };
         observe(kv_bar(0), 0, 0);
-        for (int j = 0; j < n_tiles; ++j) {
-            observe(smem_u32(&bars->p_full[0]), j & 1, 2000 + j);
-            if (j + 1 < n_tiles) observe(kv_bar(j + 1), ((j + 1) >> 2) & 1, 2 * (j + 1));
-            if (ng == 2) observe(smem_u32(&bars->p_full[1]), j & 1, 3000 + j);
-        }
+        for (int j = 0; j + 1 < n_tiles; ++j)
+            observe(kv_bar(j + 1), ((j + 1) >> 2) & 1, 2 * (j + 1));
       }
     } else {
         asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsSm));
@@ -413,12 +416,20 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
         }
         float m_run = -INFINITY;
         float l_run = 0.0f;
-        for (int j = 0; j < n_tiles && ok; ++j) {
+        // Every step ends with this group meeting the MMA warp at its P barrier (named
+        // barrier 5 + g: these 128 threads and the MMA warp's 32): the MMA warp waits on it
+        // in hardware, no mbarrier and no observer in between. Both sides pass it once per
+        // KV step whatever happens: after an error the group keeps passing without
+        // computing (a bar.sync, not an arrive, so it can never run a phase ahead). A group
+        // with no rows (the second tile of a one-tile item) takes no part: the MMA warp does
+        // not issue for it.
+        const int p_steps = active ? n_tiles : 0;
+        for (int j = 0; j < p_steps; ++j) {
+          if (ok) {
             ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&bars->s_full[g]), j & 1, lim, abort));
-            if (!ok) {
-                report(p.status, abort, 2 + g, j);
-                break;
-            }
+            if (!ok) report(p.status, abort, 2 + g, j);
+          }
+          if (ok) {
             tc_fence_after();
             float s[kBN];
             {
@@ -521,7 +532,8 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
             l_run = l_run * alpha + row_sum();
             tmem_st_wait();
             tc_fence_before();
-            mbar_arrive(smem_u32(&bars->p_full[g]));
+          }
+          named_bar_sync(kBarP + g, 160);
         }
         // ---- epilogue ------------------------------------------------------------------
         // O leaves through shared memory and TMA tensor stores. Once both tiles' last PV
