@@ -233,7 +233,7 @@ def run_gpu(args, wl, world, rank, local):
     achieved = flops / (attn_mean * 1e-3) / 1e12
 
     # e2e through the host-buffer entry point: H2D of q,k,v + step + D2H of out
-    n_e2e = max(3, min(n, 200))
+    n_e2e = max(50, min(n, 200))
     hq, hk, hv = (t.pin_memory() for t in synth.chunk_qkv(wl, sid, 1000))
     hout = torch.empty(st.shape(), dtype=torch.float32).pin_memory()
     for _ in range(2):
@@ -244,11 +244,12 @@ def run_gpu(args, wl, world, rank, local):
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
-    w0 = time.perf_counter()
-    for _ in range(n_e2e):
-        st.chunk_step_host(hq, hk, hv, hout)
-    st.sync()
-    e2e_ms = max_over_ranks((time.perf_counter() - w0) * 1e3, world, dev)
+    with ClockSampler(local) as clk_e2e:
+        w0 = time.perf_counter()
+        for _ in range(n_e2e):
+            st.chunk_step_host(hq, hk, hv, hout)
+        st.sync()
+        e2e_ms = max_over_ranks((time.perf_counter() - w0) * 1e3, world, dev)
     e2e_value = flops * n_e2e * world / (e2e_ms * 1e-3) / 1e12
     per_chunk = per_chunk_leg(st, wl, sid, dev, stream, local) if wl.chunks > wl.window else None
     st.close()
@@ -284,7 +285,8 @@ def run_gpu(args, wl, world, rank, local):
         "e2e": {"value": round(e2e_value, 2), "unit": UNIT,
                 "h2d_bytes_per_step": 3 * wl.n_q * wl.heads * wl.head_dim * 2,
                 "d2h_bytes_per_step": wl.n_q * wl.heads * wl.head_dim * 4,
-                "steps": n_e2e, "ms_per_step": round(e2e_ms / n_e2e, 4)},
+                "steps": n_e2e, "ms_per_step": round(e2e_ms / n_e2e, 4),
+                "clocks": clk_e2e.summary()},
         "gpu_launches": 2 * n,
     }
     if per_chunk is not None:
