@@ -229,10 +229,34 @@ frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w,
  * for CTA pairs (tcgen05 cta_group::2, two pixel tiles per pair) or 0 for single
  * CTAs; bn = 0 restores the automatic choice (a cost model of the launch). Applies
  * to later frt_conv_step calls, which return FRT_ERR_UNSUPPORTED for bn = 96 with a
- * bf16 output (staged in 64-channel units). Results do not depend on the tile: each
- * output sums its products in one order (temporal tap, channel block, spatial tap).
- * FRT_ERR_INVALID_ARG for other values. */
+ * bf16 output (staged in 64-channel units). With whole tiles (frt_conv_set_split
+ * mode 1) results do not depend on the tile: each output sums its products in one
+ * order (temporal tap, channel block, spatial tap). FRT_ERR_INVALID_ARG for other
+ * values; may allocate the split workspace (FRT_ERR_OOM). */
 frt_status frt_conv_set_tile(frt_conv_t* c, int bn, int pair);
+/* Work split of the convolution kernel, for tuning and tests (no counterpart in the
+ * paper). The K loop of an output tile is its halos (temporal tap x 64-channel
+ * block); the launch's units (CTAs, or CTA pairs) either take whole tiles or, split,
+ * equal shares of all tiles' halo steps in order, so that a tile's K sum may come in
+ * parts from consecutive units: each part is written to a workspace and the part that
+ * arrives last adds them in step order, then the bias. mode 0 = automatic (split
+ * when the tiles do not fill the units evenly and the cost model favours it), 1 =
+ * whole tiles only, 2 = split whenever the units do not divide the tiles; units = 0
+ * for every SM (or SM pair), else at most that many units. Results are deterministic
+ * for a given plan; split and whole-tile plans may differ in the last bits (another
+ * fp32 summation grouping, within the same error bound). Applies to later
+ * frt_conv_step calls; may allocate the workspace (FRT_ERR_OOM). FRT_ERR_INVALID_ARG
+ * for a mode outside 0..2 or units < 0. */
+frt_status frt_conv_set_split(frt_conv_t* c, int mode, int units);
+/* The launch plan frt_conv_step would use for these sizes on a GPU with `sms` SMs
+ * (host-only, launches nothing): bn and pair as frt_conv_set_tile (0 = automatic),
+ * split_mode and units as frt_conv_set_split. Writes plan[0..5] = tile width, pair
+ * (0/1), units (CTAs or CTA pairs in the grid), split (0/1), number of output tiles
+ * (pair tiles count once), halos per tile (the K steps: kt x Cin / 64).
+ * FRT_ERR_INVALID_ARG on invalid sizes, FRT_ERR_UNSUPPORTED if no tile fits. */
+frt_status frt_conv_plan(int cin, int cout, int kt, int kh, int kw, int grid_h, int grid_w,
+                         int frames_per_chunk, int out_dtype, int sms, int bn, int pair,
+                         int split_mode, int units, int* plan);
 /* The current cache [kt-1, H, W, Cin] bf16 (device, read-only use). */
 frt_status frt_conv_cache(const frt_conv_t* c, const void** cache);
 /* Wait for the handle's work; returns FRT_ERR_TIMEOUT if a device wait gave up. */

@@ -63,6 +63,9 @@ constexpr int kMaxStages = 8;
 constexpr int kTimeoutCode = 6;  // FRT_ERR_TIMEOUT
 constexpr int kSmemBudget = 225 * 1024;  // dynamic shared memory of the kernel
 constexpr int kSlab = kBM * 128;         // epilogue staging: 128 rows of 128 bytes
+// How long the first part of a split tile waits, with its own sum done, for the other
+// parts before it writes itself out instead (they usually land within a few us).
+constexpr unsigned long long kPartWaitNs = 20000;
 
 struct ConvParams {
     CUtensorMap x_map;      // 4D (Cin, W, H, F) bf16 over the chunk, box (64, halo_w, halo_h, 1)
@@ -89,6 +92,18 @@ struct ConvParams {
     uint4* shift_next;
     long long shift_frame_vec;   // vectors per frame
     int shift_keep;              // kt - 1
+    // Work split over the grid's units (a CTA, or a CTA pair): the K loop of tile t is
+    // its halos, global steps [t * nhalo, (t + 1) * nhalo). Split: unit u takes the steps
+    // [u * total / units, (u + 1) * total / units), so a tile may be shared by
+    // consecutive units, each adding a part of its K sum. Not split: unit u takes the
+    // whole tiles [u * n_tiles / units, (u + 1) * n_tiles / units).
+    long long total;             // n_tiles * nhalo
+    int split;
+    // split tiles: each part is written to part[slot][rank][BN / 4][128] (float4, slot
+    // 2u for the first item of unit u's range, 2u + 1 for its last), and the part that
+    // arrives last at counters[t * pair + rank] adds all parts in step order
+    float4* part;
+    int* counters;               // zero between launches: the adding part resets it
 };
 
 template <int BN, bool PAIR>
@@ -107,8 +122,11 @@ struct CBars {
     uint64_t acc_full[2];
     uint64_t acc_empty[2];
     uint64_t drain;
+    uint64_t part_full;     // a split tile's part copied into the (idle) rings
+    float4 bias[64];        // epilogue: the current tile's bias slice (BN <= 256)
     uint32_t tmem_base;
     int abort_flag;
+    int last_part;          // epilogue: broadcast word of the split-tile protocol
 };
 
 __device__ __forceinline__ void report(DeviceStatus* st, volatile int* abort, int role, int where) {
@@ -138,6 +156,103 @@ __device__ __forceinline__ void tile_coords(const ConvParams& p, int t, int cm, 
     f = m / p.tiles_h;
 }
 
+// First global step of unit u's share.
+__device__ __forceinline__ long long unit_start(const ConvParams& p, int u, int units, int nhalo) {
+    return p.split ? (long long)u * p.total / units : (long long)u * p.n_tiles / units * nhalo;
+}
+
+// Split: the unit whose share holds global step s (the largest u with unit_start <= s).
+__device__ __forceinline__ int unit_of(const ConvParams& p, long long s, int units) {
+    return int(((s + 1) * units - 1) / p.total);
+}
+
+// Workspace slot of unit u's part of the split tile that starts at step ts: the tile is
+// the unit's first item if its share starts inside the tile, else its last.
+__device__ __forceinline__ int part_slot(const ConvParams& p, int u, long long ts, int units,
+                                         int nhalo) {
+    return 2 * u + (unit_start(p, u, units, nhalo) < ts ? 1 : 0);
+}
+
+// The items of a unit's share in order: tile t, halos [h0, h1) of its K loop.
+struct Items {
+    long long s, s1;
+    int nhalo;
+    int t, h0, h1;
+    __device__ __forceinline__ bool next() {
+        if (s >= s1) return false;
+        t = int(s / nhalo);
+        const long long ts = (long long)t * nhalo;
+        const long long te = ts + nhalo;
+        h0 = int(s - ts);
+        h1 = int((s1 < te ? s1 : te) - ts);
+        s = ts + h1;
+        return true;
+    }
+};
+
+// Split tiles sum their parts in one order, whoever adds them: the parts that continue
+// the tile (1, 2, ..., n - 1, in step order) and then the part that starts it (0):
+// ((part 1 + part 2) + ...) + part 0. Its starting part is its unit's last item, so it
+// usually completes last, and this order lets that unit add the others while its own
+// MMAs still run.
+//
+// sum_parts: TMEM columns [dst, dst + BN) of this thread's lane become the sum, in that
+// order, of NO parts read from L2 (src[0..NO), this thread's row of each) and, at
+// position own of the order, this CTA's own part already in dst (own = -1: none). The
+// parts are read in batches of 16 16-byte loads per thread: an L2 round trip here
+// is about a microsecond, so one 32-column batch at a time would cost one per batch.
+// (Not inlined: its loads would otherwise be allocated together with the callers' live
+// state, and the epilogue would spill.)
+template <int NO, int BN>
+__device__ __noinline__ void sum_parts(uint32_t dst, const float4* const (&src)[4], int own) {
+    constexpr int CPB = (2 / NO) > 0 ? 2 / NO : 1;   // 32-column chunks per batch
+#pragma unroll 1
+    for (int c0 = 0; c0 < BN; c0 += 32 * CPB) {
+        float4 q[CPB][NO][8];
+#pragma unroll
+        for (int cb = 0; cb < CPB; ++cb)
+            if (c0 + cb * 32 < BN)
+#pragma unroll
+                for (int o = 0; o < NO; ++o)
+#pragma unroll
+                    for (int i = 0; i < 8; ++i)
+                        q[cb][o][i] = __ldcg(src[o] + size_t((c0 + cb * 32) / 4 + i) * kBM);
+#pragma unroll
+        for (int cb = 0; cb < CPB; ++cb) {
+            if (c0 + cb * 32 >= BN) break;
+            uint32_t r[32];
+            if (own >= 0) {
+                tmem_ld32(dst + uint32_t(c0 + cb * 32), r);
+                tmem_ld_wait();
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const float4 mine = make_float4(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1]),
+                                                __uint_as_float(r[4 * i + 2]), __uint_as_float(r[4 * i + 3]));
+                float4 sum = own == 0 ? mine : q[cb][0][i];
+#pragma unroll
+                for (int k = 1; k <= NO; ++k) {
+                    if (own < 0 && k == NO) break;          // NO positions without an own part
+                    // position k of the order: the own part, else global part k or k - 1
+                    const float4 a = q[cb][k < NO ? k : NO - 1][i];
+                    const float4 b = q[cb][k - 1][i];
+                    const float4 v = k == own ? mine : ((own < 0 || k < own) ? a : b);
+                    sum.x += v.x;
+                    sum.y += v.y;
+                    sum.z += v.z;
+                    sum.w += v.w;
+                }
+                r[4 * i] = __float_as_uint(sum.x);
+                r[4 * i + 1] = __float_as_uint(sum.y);
+                r[4 * i + 2] = __float_as_uint(sum.z);
+                r[4 * i + 3] = __float_as_uint(sum.w);
+            }
+            tmem_st32(dst + uint32_t(c0 + cb * 32), r);
+        }
+    }
+    tmem_st_wait();
+}
+
 template <int BN, bool PAIR>
 __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant__ ConvParams p) {
     using C = CCfg<BN, PAIR>;
@@ -159,8 +274,10 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     const uint64_t lim = p.wait_limit_ns;
     const int rank = PAIR ? int(cluster_ctarank()) : 0;
     const bool leader = rank == 0;
-    const int c_first = blockIdx.x / CM;
-    const int c_stride = gridDim.x / CM;
+    const int unit = blockIdx.x / CM;
+    const int units = gridDim.x / CM;
+    const long long s_begin = unit_start(p, unit, units, nhalo);
+    const long long s_end = unit_start(p, unit + 1, units, nhalo);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < p.a_stages; ++s) {
@@ -176,6 +293,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
             mbar_init(smem_u32(&bars.acc_empty[b]), 128 * CM);
         }
         mbar_init(smem_u32(&bars.drain), 1);
+        mbar_init(smem_u32(&bars.part_full), 1);
         bars.abort_flag = 0;
         fence_mbar_init();
     }
@@ -206,14 +324,16 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
             uint32_t ph = 0;
             int ia = 0;
             bool ok = true;
-            for (int t = c_first; t < p.n_tiles && ok; t += c_stride) {
+            Items it{s_begin, s_end, nhalo, 0, 0, 0};
+            while (ok && it.next()) {
                 int f, th, tw, tn;
-                tile_coords(p, t, CM, rank, f, th, tw, tn);
+                tile_coords(p, it.t, CM, rank, f, th, tw, tn);
                 const int cx = tw * kTileW - p.kw / 2;
                 const int cy = th * kTileH - p.kh / 2;
-                int src = f - (p.kt - 1);                 // frame of (cache, chunk) - cache
-                int kb = 0;
-                for (int hi = 0; hi < nhalo; ++hi, ++ia) {
+                // halo hi = (temporal tap hi / nkb, channel block hi % nkb)
+                int src = f - (p.kt - 1) + it.h0 / nkb;  // frame of (cache, chunk) - cache
+                int kb = it.h0 % nkb;
+                for (int hi = it.h0; hi < it.h1; ++hi, ++ia) {
                     if (ia >= p.a_stages && !mbar_test_wait(smem_u32(&bars.a_empty[s]), ph ^ 1) &&
                         !mbar_wait(smem_u32(&bars.a_empty[s]), ph ^ 1, lim, abort)) {
                         report(p.status, abort, 0, ia);
@@ -253,10 +373,12 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
             uint32_t ph = 0;
             int ib = 0;
             bool ok = true;
-            for (int t = c_first; t < p.n_tiles && ok; t += c_stride) {
-                const int n0 = (t % p.tiles_n) * BN + rank * (BN / CM);
-                int kb = 0, tap0 = 0;                     // tap0 = first tap of this dt
-                for (int hi = 0; hi < nhalo && ok; ++hi) {
+            Items it{s_begin, s_end, nhalo, 0, 0, 0};
+            while (ok && it.next()) {
+                const int n0 = (it.t % p.tiles_n) * BN + rank * (BN / CM);
+                int kb = it.h0 % nkb;
+                int tap0 = (it.h0 / nkb) * sp;            // first tap of this temporal tap
+                for (int hi = it.h0; hi < it.h1 && ok; ++hi) {
                     for (int g = 0; g < ngrp; ++g, ++ib) {
                         if (ib >= p.b_stages && !mbar_test_wait(smem_u32(&bars.b_empty[s]), ph ^ 1) &&
                             !mbar_wait(smem_u32(&bars.b_empty[s]), ph ^ 1, lim, abort)) {
@@ -313,12 +435,13 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
             const uint32_t b_step = uint32_t(p.b_stage >> 4);
             int sa = 0, sb = 0;
             int tl = 0;
-            for (int t = c_first; t < p.n_tiles; t += c_stride, ++tl) {
+            Items it{s_begin, s_end, nhalo, 0, 0, 0};
+            for (; it.next(); ++tl) {
                 const int b = tl & 1;
                 if (tl >= 2) handoff();                      // accumulator b drained
                 const uint32_t d = tmem + uint32_t(b * BN);
                 uint32_t accumulate = 0;
-                for (int hi = 0; hi < nhalo; ++hi) {
+                for (int hi = it.h0; hi < it.h1; ++hi) {
                     handoff();                               // halo stage sa landed
                     uint64_t da = da0 + uint64_t(uint32_t(sa) * a_step);
                     // a weight stage holds tb consecutive taps of one kernel row: one
@@ -373,10 +496,11 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
             uint32_t pa = 0, pb = 0;
             int ia = 0, ib = 0;
             int tl = 0;
-            for (int t = c_first; t < p.n_tiles; t += c_stride, ++tl) {
+            Items it{s_begin, s_end, nhalo, 0, 0, 0};
+            for (; it.next(); ++tl) {
                 const int b = tl & 1;
                 if (tl >= 2) observe(smem_u32(&bars.acc_empty[b]), ((tl >> 1) - 1) & 1, 1, -1 - tl);
-                for (int hi = 0; hi < nhalo; ++hi, ++ia) {
+                for (int hi = it.h0; hi < it.h1; ++hi, ++ia) {
                     observe(smem_u32(&bars.a_full[sa]), pa, 1, ia);
                     for (int dh = 0; dh < p.kh; ++dh)
                         for (int dw = 0; dw < p.kw; dw += p.tb, ++ib) {
@@ -398,16 +522,15 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
         const int sub = warp & 3;
         const int row = sub * 32 + lane;                 // pixel of the tile: 8 per row
         const uint32_t lane_off = uint32_t(sub * 32) << 16;
-        const uint32_t rb = sStg + uint32_t(row * 128);
         const uint32_t sw = uint32_t(row & 7);
         const bool est = threadIdx.x == 64;              // issues the tile's TMA stores
         const int ucols = p.y_bf16 ? 64 : 32;            // output channels per unit
         if (p.shift_keep > 0) {
             // this CTA's slice of the next cache, while the first tile's MMAs run
-            const long long total = p.shift_frame_vec * p.shift_keep;
-            const long long per = (total + gridDim.x - 1) / gridDim.x;
+            const long long nvec = p.shift_frame_vec * p.shift_keep;
+            const long long per = (nvec + gridDim.x - 1) / gridDim.x;
             const long long lo = per * blockIdx.x;
-            const long long hi = lo + per < total ? lo + per : total;
+            const long long hi = lo + per < nvec ? lo + per : nvec;
             for (long long i = lo + (threadIdx.x - 64); i < hi; i += 128) {
                 const int j = int(i / p.shift_frame_vec);
                 const long long r = i - (long long)j * p.shift_frame_vec;
@@ -418,10 +541,95 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
             }
         }
         int tl = 0;
-        for (int t = c_first; t < p.n_tiles; t += c_stride, ++tl) {
+        uint32_t part_phase = 0;                          // parity of bars.part_full
+        Items it{s_begin, s_end, nhalo, 0, 0, 0};
+        for (; it.next(); ++tl) {
             const int b = tl & 1;
             int f, th, tw, tn;
-            tile_coords(p, t, CM, rank, f, th, tw, tn);
+            tile_coords(p, it.t, CM, rank, f, th, tw, tn);
+            // the tile's bias slice, read once (the barriers below pass before its use, and
+            // the previous tile's last use precedes a barrier every thread has passed)
+            if (row < BN / 4) bars.bias[row] = __ldg(reinterpret_cast<const float4*>(p.bias + tn * BN) + row);
+            const uint32_t acc = tmem + lane_off + uint32_t(b * BN);
+            const uint32_t acc2 = tmem + lane_off + uint32_t((b ^ 1) * BN);   // the idle buffer
+            // A split tile: its parts come from units first .. first + n_parts - 1 (part
+            // k = unit - first covers the k-th piece of its halo steps) and are summed as
+            // ((part 1 + ... + part n-1) + part 0).
+            const bool split = it.h0 != 0 || it.h1 != nhalo;
+            int n_parts = 1, first = unit;
+            long long ts = 0;
+            int* ctr = nullptr;
+            if (split) {
+                ts = (long long)it.t * nhalo;
+                first = unit_of(p, ts, units);
+                n_parts = unit_of(p, ts + nhalo - 1, units) - first + 1;
+                ctr = p.counters + size_t(it.t) * CM + rank;
+            }
+            const int kpart = unit - first;
+            if (n_parts > 3) {                               // excluded by the plan
+                if (est) report(p.status, abort, 5, it.t);
+                break;
+            }
+            auto part_row = [&](int k) {                     // this thread's row of part k
+                return p.part + (size_t(part_slot(p, first + k, ts, units, nhalo)) * CM + rank) *
+                                    (BN / 4) * kBM + row;
+            };
+            auto other = [&](int j) -> const float4* {       // j-th other part in sum order
+                const int k = kpart == 0 ? j + 1 : (j < kpart - 1 ? j + 1 : (j < n_parts - 2 ? j + 2 : 0));
+                return part_row(k);
+            };
+            // TMEM dst = the sum of the other parts and, at position own of the order (-1:
+            // none), this CTA's part already in dst
+            auto sum_into = [&](uint32_t dst, int own) {
+                const int no = n_parts - 1;
+                // the plan gives every unit at least half a tile of steps: <= 3 parts
+                const float4* src[4];
+#pragma unroll
+                for (int o = 0; o < 4; ++o) src[o] = o < no ? other(o) : nullptr;
+                if (no == 1) sum_parts<1, BN>(dst, src, own);
+                else sum_parts<2, BN>(dst, src, own);
+            };
+            // Part 0 is this unit's last item. While its MMAs run, watch the tile's arrival
+            // word (part k sets bit k): every other part that has arrived is added into the
+            // idle buffer at once, so that part 0 adds itself at the end with no round trip
+            // through memory. With at most two other parts their sum is the same in either
+            // arrival order (two-operand addition commutes). Nothing waits on another CTA:
+            // the watch ends when this CTA's accumulator is ready, and whatever has not
+            // arrived by then goes the write-and-arrive way below.
+            const int others = (1 << n_parts) - 2;           // bits of parts 1 .. n-1
+            int loaded = 0;                                   // parts summed into acc2
+            auto take = [&](int fresh) {                      // add newly arrived parts
+                __threadfence();
+                const float4* src[4] = {nullptr, nullptr, nullptr, nullptr};
+                if (fresh == 6) {                             // parts 1 and 2 together
+                    src[0] = part_row(1);
+                    src[1] = part_row(2);
+                    sum_parts<2, BN>(acc2, src, -1);
+                } else {                                      // one part: the first, or added
+                    src[0] = part_row((fresh & 2) ? 1 : 2);
+                    sum_parts<1, BN>(acc2, src, loaded != 0 ? 0 : -1);
+                }
+                loaded |= fresh;
+            };
+            if (split && kpart == 0) {
+                const uint64_t t0 = globaltimer_ns();
+                for (;;) {
+                    if (est) {
+                        int st = ld_acquire_gpu(ctr) & others;
+                        if (mbar_test_wait(smem_u32(&bars.acc_full[b]), (tl >> 1) & 1)) st |= 1 << 16;
+                        else if (*abort != 0 || globaltimer_ns() - t0 > lim) st |= 1 << 17;
+                        bars.last_part = st;
+                    }
+                    named_bar_sync(1, 128);
+                    const int st = *reinterpret_cast<volatile int*>(&bars.last_part);
+                    named_bar_sync(1, 128);
+                    if ((st >> 16) != 0) break;                // accumulator ready: bulk path
+                    const int fresh = st & others & ~loaded;
+                    if (fresh != 0) take(fresh);
+                    if (loaded == others) break;
+                    __nanosleep(500);
+                }
+            }
             const bool got = mbar_wait(smem_u32(&bars.acc_full[b]), (tl >> 1) & 1, lim, abort);
             // all four warps go on or stop together: the staging below synchronises them
             if (!named_bar_and(1, 128, got)) {
@@ -429,6 +637,130 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
                 break;
             }
             tc_fence_after();
+            bool early_ready = false;
+            if (split && kpart == 0) {
+                // Part 0, accumulator ready: the parts still missing are usually a few
+                // microseconds from arriving (a unit whose whole share lies inside this tile
+                // ends when this one does). Give them kPartWaitNs, taking each as it lands;
+                // reading one part then is cheaper than writing this one and having the
+                // last arrival read them all. Past that, write and arrive as below.
+                // This is the unit's last item, so its MMAs are done and the halo and
+                // weight rings are idle: a part that lands now is brought in by bulk copies
+                // (16 KB per 32 columns) and added from shared memory, which keeps many
+                // more bytes in flight than loads into registers can.
+                const uint32_t ring_bytes = uint32_t(p.a_stages * p.a_bytes + p.b_stages * p.b_stage);
+                const bool bulk = ring_bytes >= uint32_t(kBM * BN * 4);
+                const uint64_t t0 = globaltimer_ns();
+                bool bad = false;
+                while (loaded != others && !bad) {
+                    if (est) {
+                        int st = ld_acquire_gpu(ctr) & others;
+                        if (*abort != 0 || globaltimer_ns() - t0 > kPartWaitNs) st |= 1 << 16;
+                        bars.last_part = st;
+                    }
+                    named_bar_sync(1, 128);
+                    const int st = *reinterpret_cast<volatile int*>(&bars.last_part);
+                    named_bar_sync(1, 128);
+                    const int fresh = st & others & ~loaded;
+                    if (fresh != 0 && !bulk) take(fresh);
+                    for (int k = 1; bulk && k < n_parts; ++k) {
+                        if ((fresh & (1 << k)) == 0) continue;
+                        const float4* blk = p.part + (size_t(part_slot(p, first + k, ts, units, nhalo)) * CM + rank) *
+                                                         (BN / 4) * kBM;
+                        if (est) {
+                            fence_proxy_async_global();
+                            mbar_arrive_expect_tx(smem_u32(&bars.part_full), uint32_t(kBM * BN * 4));
+                            for (int c = 0; c < BN; c += 32)
+                                bulk_load(sA + uint32_t(c * kBM * 4), blk + size_t(c / 4) * kBM,
+                                          uint32_t(32 * kBM * 4), smem_u32(&bars.part_full));
+                        }
+                        const bool in = __all_sync(0xffffffffu, mbar_wait(smem_u32(&bars.part_full), part_phase, lim, abort));
+                        part_phase ^= 1;
+                        if (!named_bar_and(1, 128, in)) {
+                            if (est) report(p.status, abort, 6, it.t);
+                            bad = true;
+                            break;
+                        }
+                        // acc2 = that part (the first taken) or acc2 + it (two-operand sums
+                        // commute, so the arrival order does not matter)
+#pragma unroll 1
+                        for (int c = 0; c < BN; c += 32) {
+                            uint32_t r[32];
+                            if (loaded != 0) {
+                                tmem_ld32(acc2 + uint32_t(c), r);
+                                tmem_ld_wait();
+                            }
+#pragma unroll
+                            for (int i = 0; i < 8; ++i) {
+                                const uint4 q = ld_shared_v4(sA + uint32_t(((c / 4 + i) * kBM + row) * 16));
+                                if (loaded != 0) {
+                                    r[4 * i] = __float_as_uint(__uint_as_float(r[4 * i]) + __uint_as_float(q.x));
+                                    r[4 * i + 1] = __float_as_uint(__uint_as_float(r[4 * i + 1]) + __uint_as_float(q.y));
+                                    r[4 * i + 2] = __float_as_uint(__uint_as_float(r[4 * i + 2]) + __uint_as_float(q.z));
+                                    r[4 * i + 3] = __float_as_uint(__uint_as_float(r[4 * i + 3]) + __uint_as_float(q.w));
+                                } else {
+                                    r[4 * i] = q.x;
+                                    r[4 * i + 1] = q.y;
+                                    r[4 * i + 2] = q.z;
+                                    r[4 * i + 3] = q.w;
+                                }
+                            }
+                            tmem_st32(acc2 + uint32_t(c), r);
+                        }
+                        tmem_st_wait();
+                        loaded |= 1 << k;
+                        named_bar_sync(1, 128);               // the ring is read before the next copy
+                    }
+                    if ((st >> 16) != 0) break;
+                    if (loaded != others && !bad) __nanosleep(256);
+                }
+                if (bad) break;
+                early_ready = loaded == others;
+                if (early_ready && est) *ctr = 0;             // parts 1 .. n-1 arrived, 0 did not
+            }
+            if (split && !early_ready) {
+                // any other case: the part is written out and counted, and the one that
+                // completes the count adds them all
+                bool adder;
+                {
+                    float4* mine = part_row(kpart);
+#pragma unroll 1
+                    for (int c = 0; c < BN; c += 32) {
+                        uint32_t r[32];
+                        tmem_ld32(acc + uint32_t(c), r);
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int i = 0; i < 8; ++i)
+                            mine[size_t(c / 4 + i) * kBM] =
+                                make_float4(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1]),
+                                            __uint_as_float(r[4 * i + 2]), __uint_as_float(r[4 * i + 3]));
+                    }
+                    named_bar_sync(1, 128);
+                    if (est) {
+                        // publishes the part (every thread's stores precede the barrier)
+                        const int bit = 1 << kpart;
+                        const int old = atom_add_acq_rel_gpu(ctr, bit);
+                        const int last = old + bit == (1 << n_parts) - 1;
+                        if (last) *ctr = 0;                  // every part has arrived
+                        bars.last_part = last;
+                    }
+                    named_bar_sync(1, 128);
+                    adder = *reinterpret_cast<volatile int*>(&bars.last_part) != 0;
+                    named_bar_sync(1, 128);
+                }
+                if (!adder) {
+                    tc_fence_before();
+                    if (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&bars.acc_empty[b]), 0));
+                    else mbar_arrive(smem_u32(&bars.acc_empty[b]));
+                    continue;
+                }
+                __threadfence();                             // the other parts are visible
+                sum_into(acc, kpart == 0 ? n_parts - 1 : kpart - 1);
+            }
+            // On the unit's last item the rings are idle: every column unit gets its own
+            // slab there and the stores go out together, instead of one slab in turn.
+            const bool wide = it.s >= s_end &&
+                              p.a_stages * p.a_bytes + p.b_stages * p.b_stage >= (BN / ucols) * kSlab;
 #pragma unroll 1
             for (int u = 0; u < BN / ucols; ++u) {
                 // the unit's 32 words per thread are computed before the slab is claimed,
@@ -439,17 +771,24 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
                     if (h == 1 && !p.y_bf16) break;
                     const int c = u * ucols + h * 32;    // first column of this TMEM load
                     uint32_t r[32];
-                    tmem_ld32(tmem + lane_off + uint32_t(b * BN + c), r);
+                    tmem_ld32(acc + uint32_t(c), r);
                     tmem_ld_wait();
-                    const float4* bp = reinterpret_cast<const float4*>(p.bias + tn * BN + c);
                     float v[32];
 #pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+                    if (early_ready) {                       // (parts 1 .. n-1) + part 0
+                        tmem_ld32(acc2 + uint32_t(c), r);
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]) + v[i];
+                    }
+#pragma unroll
                     for (int i = 0; i < 8; ++i) {
-                        const float4 bb = __ldg(bp + i);
-                        v[4 * i] = __uint_as_float(r[4 * i]) + bb.x;
-                        v[4 * i + 1] = __uint_as_float(r[4 * i + 1]) + bb.y;
-                        v[4 * i + 2] = __uint_as_float(r[4 * i + 2]) + bb.z;
-                        v[4 * i + 3] = __uint_as_float(r[4 * i + 3]) + bb.w;
+                        const float4 bb = bars.bias[c / 4 + i];
+                        v[4 * i] += bb.x;
+                        v[4 * i + 1] += bb.y;
+                        v[4 * i + 2] += bb.z;
+                        v[4 * i + 3] += bb.w;
                     }
                     if (p.y_bf16) {
 #pragma unroll
@@ -459,16 +798,32 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
                         for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(v[i]);
                     }
                 }
-                if (est) bulk_wait_read<0>();            // the previous store has read the slab
-                named_bar_sync(1, 128);
+                const uint32_t slab = wide ? sA + uint32_t(u * kSlab) : sStg;
+                if (!wide) {
+                    if (est) bulk_wait_read<0>();        // the previous store has read the slab
+                    named_bar_sync(1, 128);
+                }
+                const uint32_t rbu = slab + uint32_t(row * 128);
 #pragma unroll
                 for (int i = 0; i < 8; ++i)
-                    st_shared_v4(rb + ((uint32_t(i) ^ sw) << 4), o[4 * i], o[4 * i + 1], o[4 * i + 2],
+                    st_shared_v4(rbu + ((uint32_t(i) ^ sw) << 4), o[4 * i], o[4 * i + 1], o[4 * i + 2],
                                  o[4 * i + 3]);
+                if (!wide) {
+                    fence_proxy_async_smem();
+                    named_bar_sync(1, 128);
+                    if (est && f < p.F) {
+                        tma_store_4d(&p.y_map, sStg, tn * BN + u * ucols, tw * kTileW, th * kTileH, f);
+                        bulk_commit();
+                    }
+                }
+            }
+            if (wide) {
                 fence_proxy_async_smem();
                 named_bar_sync(1, 128);
                 if (est && f < p.F) {
-                    tma_store_4d(&p.y_map, sStg, tn * BN + u * ucols, tw * kTileW, th * kTileH, f);
+                    for (int u = 0; u < BN / ucols; ++u)
+                        tma_store_4d(&p.y_map, sA + uint32_t(u * kSlab), tn * BN + u * ucols, tw * kTileW,
+                                     th * kTileH, f);
                     bulk_commit();
                 }
             }
@@ -476,7 +831,9 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
             if (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&bars.acc_empty[b]), 0));
             else mbar_arrive(smem_u32(&bars.acc_empty[b]));
         }
-        if (est) bulk_wait<0>();                          // y written before the CTA exits
+        // the stores have read their slabs before the CTA exits (their writes complete
+        // with the grid)
+        if (est) bulk_wait_read<0>();
     }
     __syncwarp();
     tc_fence_before();
@@ -490,7 +847,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
 }
 
 template <int BN, bool PAIR>
-cudaError_t launch_conv(ConvParams p, cudaStream_t st) {
+cudaError_t launch_conv(ConvParams p, int units, cudaStream_t st) {
     using C = CCfg<BN, PAIR>;
     const int smem = p.a_stages * p.a_bytes + p.b_stages * p.b_stage + kSlab + 1024;
     static int attr[kMaxDevices] = {};   // per device: the largest size set so far
@@ -501,7 +858,6 @@ cudaError_t launch_conv(ConvParams p, cudaStream_t st) {
         if (e != cudaSuccess) return e;
         if (dev >= 0) attr[dev] = smem;
     }
-    const int units = std::min(p.n_tiles, num_sms() / C::CM);
     if (!PAIR) {
         conv_kernel<BN, false><<<units, kThreads, smem, st>>>(p);
         return cudaGetLastError();
@@ -577,41 +933,85 @@ bool plan_rings(int a_bytes, int b_bytes, int kw, int& tb, int& a_stages, int& b
     return b_stages >= 2;
 }
 
-// Output-channel tile and pairing, from a cost model measured on GB300 with this
-// kernel: a spatial tap costs its MMA issue time (four MMAs of max(BN / 2, 50) cycles,
-// 1.2x that for CTA pairs, whose MMAs issue slower) plus ~350 cycles of ring
-// bookkeeping (a shared-memory access by the issuing thread behind queued MMAs costs it
-// ~140 cycles), plus ~300 more when a weight stage holds a single tap; every tile has the
-// same number of taps and tiles run in rounds over the SMs (or SM pairs), so a launch
-// costs rounds x that. The cheapest of the widths dividing Cout wins; pairs need at
-// least two pixel tiles. A bf16 output is staged in 64-channel units, so its widths are
-// multiples of 64.
-int choose_bn(int cout, long long m_tiles, int a_bytes, int kw, bool y_bf16, bool& pair) {
+// Launch plan of one chunk: tile width, pairing, rings, units and whether tiles are split.
+struct ConvPlan {
+    int bn = 0;
+    bool pair = false;
+    int tb = 1, a_stages = 2, b_stages = 2;
+    int tiles_n = 0, n_tiles = 0;
+    int units = 0;             // CTAs, or CTA pairs
+    bool split = false;
+    long long total = 0;       // n_tiles * halos per tile
+};
+
+// Cycles per spatial tap (four MMAs of K 16 and their share of the ring hand-offs),
+// fitted to clock traces and timings of this kernel on GB300: single CTAs are bound by
+// shared-memory operand reads (A, B and the weight copies), about 3.5 cycles per output
+// channel of the tile, with a floor of about 450; CTA pairs read half of B each and
+// take about 570 cycles per tap up to BN 192. A weight stage of one tap adds about 300.
+double tap_cycles(int bn, bool pair, int tb, int kw) {
+    const double t = pair ? std::max(570.0, 2.3 * bn) : std::max(450.0, 3.5 * bn);
+    return t + (tb == 1 && kw > 1 ? 300.0 : 0.0);
+}
+
+// Cycles a split tile's last part spends beyond its MMAs: writing its part, reading the
+// others and the store (measured 1-2 us at the VAE sizes).
+constexpr double kSplitCycles = 3000.0;
+
+// split_mode: 0 automatic, 1 whole tiles only, 2 split whenever units do not divide the
+// tiles evenly. units_req: 0 = every SM (or SM pair), else at most that many units.
+// bn_req / pair_req: 0 = automatic tile. Returns false if nothing fits.
+bool plan_conv(int cin, int cout, int kt, int kh, int kw, int H, int W, int F, bool y_bf16,
+               int bn_req, int pair_req, int split_mode, int units_req, int sms, ConvPlan& out) {
+    const int halo_w = kTileW + kw - 1, halo_h = kTileH + kh - 1;
+    const int a_bytes = (halo_w * halo_h * kBK * 2 + 1023) & ~1023;
+    const long long m_tiles =
+        (long long)F * ((W + kTileW - 1) / kTileW) * ((H + kTileH - 1) / kTileH);
+    const int nhalo = kt * (cin / kBK);
+    const int sp = kh * kw;
     const int cands[5] = {256, 192, 128, 96, 64};
-    const long long sms = num_sms();
-    int best = 0;
-    double best_t = 1e30;
+    double best_t = 1e300;
+    bool found = false;
     for (int pr = 0; pr < 2; ++pr) {
-        if (pr == 1 && m_tiles < 2) continue;
+        if (bn_req != 0 && pr != pair_req) continue;
+        if (pr == 1 && m_tiles < 2 && bn_req == 0) continue;
         const int cm = pr ? 2 : 1;
-        const long long units = sms / cm;
-        const long long mt = (m_tiles + cm - 1) / cm;
+        const long long m_units = (m_tiles + cm - 1) / cm;
+        long long all = sms / cm;
+        if (units_req > 0) all = std::min<long long>(all, units_req);
         for (int bn : cands) {
+            if (bn_req != 0 && bn != bn_req) continue;
             if (cout % bn || (y_bf16 && bn % 64)) continue;
-            int tb, as, bs;
-            if (!plan_rings(a_bytes, (bn / cm) * kBK * 2, kw, tb, as, bs)) continue;
-            const long long tiles = mt * (cout / bn);
-            const double rounds = double((tiles + units - 1) / units);
-            const double mma = 4.0 * std::max(bn / 2.0, 50.0) * (pr ? 1.2 : 1.0);
-            const double t = rounds * (350.0 + mma + (tb == 1 && kw > 1 ? 300.0 : 0.0));
+            ConvPlan c;
+            c.bn = bn;
+            c.pair = pr == 1;
+            if (!plan_rings(a_bytes, (bn / cm) * kBK * 2, kw, c.tb, c.a_stages, c.b_stages)) continue;
+            c.tiles_n = cout / bn;
+            if (m_units * c.tiles_n >= (1LL << 31)) continue;
+            c.n_tiles = int(m_units * c.tiles_n);
+            c.total = (long long)c.n_tiles * nhalo;
+            const double halo = sp * tap_cycles(bn, c.pair, c.tb, kw);
+            // whole tiles in rounds over the units
+            const long long uw = std::min<long long>(all, c.n_tiles);
+            const double t_whole = double((c.n_tiles + uw - 1) / uw) * nhalo * halo;
+            // split: every unit takes an equal share of the halo steps, at least half a
+            // tile's, so that a tile has at most three parts
+            const long long us = std::min<long long>(all, c.total / ((nhalo + 1) / 2));
+            const double t_split = double((c.total + us - 1) / us) * halo + kSplitCycles;
+            const bool uneven = c.n_tiles % uw != 0 || uw < all;
+            c.split = split_mode == 2 ? (c.n_tiles % us != 0 || us > c.n_tiles)
+                    : split_mode == 1 ? false
+                                      : (uneven && t_split < t_whole);
+            c.units = int(c.split ? us : uw);
+            const double t = c.split ? t_split : t_whole;
             if (t < best_t - 1e-9) {
                 best_t = t;
-                best = bn;
-                pair = pr == 1;
+                out = c;
+                found = true;
             }
         }
     }
-    return best;
+    return found;
 }
 
 }  // namespace
@@ -633,6 +1033,14 @@ struct frt_conv {
     unsigned long long wait_limit_ns = 2000000000ull;
     int force_bn = 0;      // 0: the cost model picks the tile
     int force_pair = 0;
+    int split_mode = 0;    // 0 automatic, 1 whole tiles, 2 split when uneven
+    int split_units = 0;   // 0: every SM (or SM pair)
+    // split tiles: parts [2 * units][pair][BN][128] fp32 and one arrival counter per
+    // tile and pair rank, sized for the current plan
+    void* part = nullptr;
+    size_t part_bytes = 0;
+    int* counters = nullptr;
+    size_t n_counters = 0;
 };
 
 namespace {
@@ -650,8 +1058,54 @@ void free_conv(frt_conv_t* c) {
     for (int i = 0; i < 2; ++i)
         if (c->cache[i]) cudaFree(c->cache[i]);
     if (c->status_host) cudaFreeHost(c->status_host);
+    if (c->part) cudaFree(c->part);
+    if (c->counters) cudaFree(c->counters);
     c->cache[0] = c->cache[1] = nullptr;
     c->status_host = c->status_dev = nullptr;
+    c->part = nullptr;
+    c->counters = nullptr;
+    c->part_bytes = c->n_counters = 0;
+}
+
+bool conv_plan(const frt_conv_t* c, ConvPlan& pl) {
+    return plan_conv(c->cin, c->cout, c->kt, c->kh, c->kw, c->H, c->W, c->F,
+                     c->out_dtype == FRT_OUT_BF16, c->force_bn, c->force_pair, c->split_mode,
+                     c->split_units, num_sms(), pl);
+}
+
+// Size the split workspace for the current plan (grows only; synchronises before it
+// frees). Called where the plan can change: configure and the tuning setters.
+frt_status ensure_split_scratch(frt_conv_t* c) {
+    ConvPlan pl;
+    if (!conv_plan(c, pl) || !pl.split) return FRT_OK;     // step reports an unfit plan
+    const int cm = pl.pair ? 2 : 1;
+    const size_t need = size_t(2) * pl.units * cm * kBM * pl.bn * sizeof(float);
+    const size_t n_ctr = size_t(pl.n_tiles) * cm;
+    cudaError_t e = cudaSuccess;
+    if (need > c->part_bytes || n_ctr > c->n_counters) {
+        if ((e = cudaStreamSynchronize(c->cs)) != cudaSuccess) return cuda_cfail(FRT_ERR_CUDA, "sync failed");
+    }
+    if (need > c->part_bytes) {
+        if (c->part) cudaFree(c->part);
+        c->part = nullptr;
+        c->part_bytes = 0;
+        if ((e = cudaMalloc(&c->part, need)) != cudaSuccess)
+            return cuda_cfail(e == cudaErrorMemoryAllocation ? FRT_ERR_OOM : FRT_ERR_CUDA,
+                              "split workspace allocation failed");
+        c->part_bytes = need;
+    }
+    if (n_ctr > c->n_counters) {
+        if (c->counters) cudaFree(c->counters);
+        c->counters = nullptr;
+        c->n_counters = 0;
+        if ((e = cudaMalloc(&c->counters, n_ctr * sizeof(int))) != cudaSuccess ||
+            (e = cudaMemset(c->counters, 0, n_ctr * sizeof(int))) != cudaSuccess ||
+            (e = cudaDeviceSynchronize()) != cudaSuccess)
+            return cuda_cfail(e == cudaErrorMemoryAllocation ? FRT_ERR_OOM : FRT_ERR_CUDA,
+                              "split counter allocation failed");
+        c->n_counters = n_ctr;
+    }
+    return FRT_OK;
 }
 }  // namespace
 
@@ -709,7 +1163,7 @@ frt_status frt_conv_configure(frt_conv_t* c, int out_dtype, void* cuda_stream) {
     c->out_dtype = out_dtype;
     c->cs = static_cast<cudaStream_t>(cuda_stream);
     c->configured = true;
-    return FRT_OK;
+    return ensure_split_scratch(c);
 }
 
 frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w, const void* bias, void* y) {
@@ -737,22 +1191,31 @@ frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w, const void
     p.halo_h = kTileH + c->kh - 1;
     p.halo_tx = p.halo_w * p.halo_h * kBK * 2;
     p.a_bytes = (p.halo_tx + 1023) & ~1023;
-    const long long m_tiles = (long long)c->F * p.tiles_w * p.tiles_h;
-    bool pair = c->force_pair != 0;
     const bool y_bf16 = c->out_dtype == FRT_OUT_BF16;
-    const int bn = c->force_bn != 0 ? c->force_bn
-                                    : choose_bn(c->cout, m_tiles, p.a_bytes, c->kw, y_bf16, pair);
-    if (bn == 0) return cfail(FRT_ERR_UNSUPPORTED, "Cout has no supported tile width");
-    if (y_bf16 && bn % 64)
+    if (y_bf16 && c->force_bn % 64)
         return cfail(FRT_ERR_UNSUPPORTED, "a bf16 output needs a tile width that is a multiple of 64");
+    ConvPlan pl;
+    if (!conv_plan(c, pl))
+        return cfail(FRT_ERR_UNSUPPORTED, "no tile width fits Cout and the shared-memory rings");
+    const int bn = pl.bn;
+    const bool pair = pl.pair;
     const int b_bytes = (pair ? bn / 2 : bn) * kBK * 2;
-    if (!plan_rings(p.a_bytes, b_bytes, c->kw, p.tb, p.a_stages, p.b_stages))
-        return cfail(FRT_ERR_UNSUPPORTED, "halo and weight rings do not fit");
+    p.tb = pl.tb;
+    p.a_stages = pl.a_stages;
+    p.b_stages = pl.b_stages;
     p.b_stage = p.tb * b_bytes;
-    p.tiles_n = c->cout / bn;
-    const long long m_units = pair ? (m_tiles + 1) / 2 : m_tiles;
-    if (m_units * p.tiles_n >= (1LL << 31)) return cfail(FRT_ERR_UNSUPPORTED, "too many tiles");
-    p.n_tiles = int(m_units * p.tiles_n);
+    p.tiles_n = pl.tiles_n;
+    p.n_tiles = pl.n_tiles;
+    p.total = pl.total;
+    p.split = pl.split ? 1 : 0;
+    if (pl.split) {
+        const int cm = pair ? 2 : 1;
+        if (size_t(2) * pl.units * cm * kBM * bn * sizeof(float) > c->part_bytes ||
+            size_t(pl.n_tiles) * cm > c->n_counters)
+            return cfail(FRT_ERR_STATE, "split workspace missing: configure the conv again");
+        p.part = static_cast<float4*>(c->part);
+        p.counters = c->counters;
+    }
     const cuuint32_t abox[4] = {64, cuuint32_t(p.halo_w), cuuint32_t(p.halo_h), 1};
     const cuuint64_t xdims[4] = {cuuint64_t(c->cin), cuuint64_t(c->W), cuuint64_t(c->H),
                                  cuuint64_t(c->F)};
@@ -782,16 +1245,16 @@ frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w, const void
     }
     cudaError_t e;
     switch (bn * 2 + (pair ? 1 : 0)) {
-        case 513: e = launch_conv<256, true>(p, c->cs); break;
-        case 512: e = launch_conv<256, false>(p, c->cs); break;
-        case 385: e = launch_conv<192, true>(p, c->cs); break;
-        case 384: e = launch_conv<192, false>(p, c->cs); break;
-        case 257: e = launch_conv<128, true>(p, c->cs); break;
-        case 256: e = launch_conv<128, false>(p, c->cs); break;
-        case 193: e = launch_conv<96, true>(p, c->cs); break;
-        case 192: e = launch_conv<96, false>(p, c->cs); break;
-        case 129: e = launch_conv<64, true>(p, c->cs); break;
-        default: e = launch_conv<64, false>(p, c->cs); break;
+        case 513: e = launch_conv<256, true>(p, pl.units, c->cs); break;
+        case 512: e = launch_conv<256, false>(p, pl.units, c->cs); break;
+        case 385: e = launch_conv<192, true>(p, pl.units, c->cs); break;
+        case 384: e = launch_conv<192, false>(p, pl.units, c->cs); break;
+        case 257: e = launch_conv<128, true>(p, pl.units, c->cs); break;
+        case 256: e = launch_conv<128, false>(p, pl.units, c->cs); break;
+        case 193: e = launch_conv<96, true>(p, pl.units, c->cs); break;
+        case 192: e = launch_conv<96, false>(p, pl.units, c->cs); break;
+        case 129: e = launch_conv<64, true>(p, pl.units, c->cs); break;
+        default: e = launch_conv<64, false>(p, pl.units, c->cs); break;
     }
     if (e != cudaSuccess) return cuda_cfail(FRT_ERR_CUDA, cudaGetErrorString(e));
     if (c->kt > 1) c->cur ^= 1;
@@ -811,7 +1274,36 @@ frt_status frt_conv_set_tile(frt_conv_t* c, int bn, int pair) {
         return cfail(FRT_ERR_INVALID_ARG, "bn must be 64, 96, 128, 192 or 256 dividing Cout; pair 0 or 1");
     c->force_bn = bn;
     c->force_pair = pair;
+    return c->configured ? ensure_split_scratch(c) : FRT_OK;
+}
+
+frt_status frt_conv_plan(int cin, int cout, int kt, int kh, int kw, int grid_h, int grid_w,
+                         int frames_per_chunk, int out_dtype, int sms, int bn, int pair,
+                         int split_mode, int units, int* plan) {
+    if (!plan || cin < 64 || cin % 64 || cout < 64 || cout % 64 || kt < 1 || kh < 1 || kw < 1 ||
+        grid_h < 1 || grid_w < 1 || frames_per_chunk < 1 || sms < 1 || split_mode < 0 ||
+        split_mode > 2 || units < 0)
+        return cfail(FRT_ERR_INVALID_ARG, "invalid sizes or modes");
+    ConvPlan pl;
+    if (!plan_conv(cin, cout, kt, kh, kw, grid_h, grid_w, frames_per_chunk,
+                   out_dtype == FRT_OUT_BF16, bn, pair, split_mode, units, sms, pl))
+        return cfail(FRT_ERR_UNSUPPORTED, "no tile width fits");
+    plan[0] = pl.bn;
+    plan[1] = pl.pair ? 1 : 0;
+    plan[2] = pl.units;
+    plan[3] = pl.split ? 1 : 0;
+    plan[4] = pl.n_tiles;
+    plan[5] = kt * (cin / kBK);
     return FRT_OK;
+}
+
+frt_status frt_conv_set_split(frt_conv_t* c, int mode, int units) {
+    if (!c) return cfail(FRT_ERR_INVALID_ARG, "NULL conv handle");
+    if (mode < 0 || mode > 2 || units < 0)
+        return cfail(FRT_ERR_INVALID_ARG, "mode 0 (automatic), 1 (whole tiles) or 2 (split); units >= 0");
+    c->split_mode = mode;
+    c->split_units = units;
+    return c->configured ? ensure_split_scratch(c) : FRT_OK;
 }
 
 frt_status frt_conv_cache(const frt_conv_t* c, const void** cache) {
@@ -838,6 +1330,9 @@ frt_status frt_conv_reset(frt_conv_t* c) {
     cudaError_t e = cudaStreamSynchronize(c->cs);
     const size_t bytes = std::max<size_t>(1, size_t(c->kt - 1)) * c->frame_bytes;
     for (int i = 0; i < 2 && e == cudaSuccess; ++i) e = cudaMemset(c->cache[i], 0, bytes);
+    // a launch that gave up may have left split tiles half counted
+    if (e == cudaSuccess && c->counters) e = cudaMemset(c->counters, 0, c->n_counters * sizeof(int));
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) return cuda_cfail(FRT_ERR_CUDA, cudaGetErrorString(e));
     std::memset(c->status_host, 0, sizeof(DeviceStatus));
     c->cur = 0;

@@ -414,7 +414,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const __grid_constant
             if (PAIR) mbar_arrive_cluster(mapa_shared(smem_u32(&bars.acc_empty[b]), 0));
             else mbar_arrive(smem_u32(&bars.acc_empty[b]));
         }
-        if (est) bulk_wait<0>();                       // C written before the CTA exits
+        // the stores have read their slabs before the CTA exits (their writes complete
+        // with the grid)
+        if (est) bulk_wait_read<0>();
     }
     __syncwarp();
     tc_fence_before();

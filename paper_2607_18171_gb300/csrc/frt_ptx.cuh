@@ -44,6 +44,20 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 }
 
 // Non-blocking test of phase `parity` of an mbarrier (returns at once).
+// atomicAdd with acquire-release semantics at GPU scope. After a barrier of the
+// threads whose writes it publishes, one thread's release makes those writes visible to
+// whoever acquires the new value (release is cumulative over the barrier).
+__device__ __forceinline__ int atom_add_acq_rel_gpu(int* p, int v) {
+    int old;
+    asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
+// A 32-bit load with acquire semantics at GPU scope (reads L2, not a stale L1 line).
+__device__ __forceinline__ int ld_acquire_gpu(const int* p) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
 __device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(

@@ -82,6 +82,8 @@ def lib() -> ctypes.CDLL:
         "frt_conv_step": (I, [P, P, P, P, P]),
         "frt_conv_cache": (I, [P, ctypes.POINTER(P)]),
         "frt_conv_set_tile": (I, [P, I, I]),
+        "frt_conv_set_split": (I, [P, I, I]),
+        "frt_conv_plan": (I, [I, I, I, I, I, I, I, I, I, I, I, I, I, I, ctypes.POINTER(ctypes.c_int)]),
         "frt_conv_sync": (I, [P]),
         "frt_conv_reset": (I, [P]),
         "frt_conv_destroy": (None, [P]),
@@ -368,6 +370,11 @@ class ConvStream:
         """Force the kernel's output-channel tile and CTA pairing (bn = 0: automatic)."""
         _check(lib().frt_conv_set_tile(self._h, bn, pair))
 
+    def set_split(self, mode: int = 0, units: int = 0) -> None:
+        """Force the kernel's work split: 0 automatic, 1 whole tiles, 2 split tiles'
+        halo steps over the units; units = 0 for every SM (or SM pair)."""
+        _check(lib().frt_conv_set_split(self._h, mode, units))
+
     def cache(self) -> torch.Tensor:
         p = ctypes.c_void_p()
         _check(lib().frt_conv_cache(self._h, ctypes.byref(p)))
@@ -486,6 +493,18 @@ def attention_plan(n_q, n_kv, heads: int, sms: int = 0) -> tuple[int, int]:
     nf, ns = ctypes.c_int(), ctypes.c_int()
     _check(lib().frt_attention_plan(n, a, b, heads, sms, ctypes.byref(nf), ctypes.byref(ns)))
     return nf.value, ns.value
+
+
+def conv_plan(cin: int, cout: int, kt: int, kh: int, kw: int, grid_h: int, grid_w: int,
+              frames: int, sms: int, out_dtype=torch.float32, bn: int = 0, pair: int = 0,
+              split_mode: int = 0, units: int = 0) -> dict:
+    """The launch plan of frt_conv_step for these sizes on `sms` SMs (host-only)."""
+    plan = (ctypes.c_int * 6)()
+    _check(lib().frt_conv_plan(cin, cout, kt, kh, kw, grid_h, grid_w, frames,
+                               OUT_BF16 if out_dtype == torch.bfloat16 else OUT_F32, sms, bn,
+                               pair, split_mode, units, plan))
+    return dict(bn=plan[0], pair=plan[1], units=plan[2], split=plan[3], n_tiles=plan[4],
+                nhalo=plan[5])
 
 
 def gemm_bf16(a: torch.Tensor, b: torch.Tensor, c: torch.Tensor,

@@ -246,3 +246,97 @@ def test_attention_plan_checks_arguments(frt):
         frt.attention_plan([0], [10], 2)
     with pytest.raises(frt.FrtError):
         frt.attention_plan([10], [10], 0)
+
+
+# ---- convolution launch plan (host-only) -------------------------------------------
+
+def _conv_items(total, n_tiles, nhalo, units, split):
+    """The kernel's share arithmetic written out: unit u's steps, then its items (tile,
+    first halo, end halo) in order."""
+    def start(u):
+        return u * total // units if split else u * n_tiles // units * nhalo
+    out = []
+    for u in range(units):
+        s, s1 = start(u), start(u + 1)
+        while s < s1:
+            t = s // nhalo
+            ts = t * nhalo
+            h0, h1 = s - ts, min(s1, ts + nhalo) - ts
+            out.append((u, t, h0, h1, start(u) < ts))
+            s = ts + h1
+    return out
+
+
+@pytest.mark.parametrize("n_tiles,nhalo,units", [(42, 18, 76), (78, 9, 76), (126, 18, 152),
+                                                 (6, 3, 18), (2, 3, 5), (7, 4, 3), (5, 18, 76),
+                                                 (1, 1, 1), (3, 9, 27), (200, 18, 76)])
+def test_conv_split_shares_cover_every_step_once_with_distinct_part_slots(n_tiles, nhalo, units):
+    total = n_tiles * nhalo
+    units = min(units, total)
+    items = _conv_items(total, n_tiles, nhalo, units, True)
+    seen = [[0] * nhalo for _ in range(n_tiles)]
+    slots = {}
+    for u, t, h0, h1, last in items:
+        assert 0 <= h0 < h1 <= nhalo
+        for h in range(h0, h1):
+            seen[t][h] += 1
+        if (h0, h1) != (0, nhalo):
+            # contributors of a split tile: units unit_of(ts) .. unit_of(ts + nhalo - 1)
+            first = ((t * nhalo + 1) * units - 1) // total
+            lastu = (((t + 1) * nhalo) * units - 1) // total
+            assert first <= u <= lastu and lastu > first
+            slot = 2 * u + (1 if last else 0)
+            assert slot not in slots, "two parts share a workspace slot"
+            slots[slot] = (t, u)
+    assert all(c == 1 for row in seen for c in row)
+    # with every share at least half a tile (the plan's cap on units) a tile has at most
+    # three parts: the kernel adds one or two other parts
+    if units <= total // ((nhalo + 1) // 2):
+        for t in range(n_tiles):
+            first = ((t * nhalo + 1) * units - 1) // total
+            lastu = (((t + 1) * nhalo) * units - 1) // total
+            assert lastu - first + 1 <= 3
+    # only a unit's first and last items can be parts of split tiles
+    for u in range(units):
+        mine = [it for it in items if it[0] == u]
+        for k, (_, _, h0, h1, _) in enumerate(mine):
+            if 0 < k < len(mine) - 1:
+                assert (h0, h1) == (0, nhalo)
+    # whole-tile shares cover every tile once
+    whole = _conv_items(total, n_tiles, nhalo, min(units, n_tiles), False)
+    assert sorted(t for _, t, h0, h1, _ in whole if (h0, h1) == (0, nhalo)) == list(range(n_tiles))
+    assert all((h0, h1) == (0, nhalo) for _, _, h0, h1, _ in whole)
+
+
+def test_conv_plan_worked_examples(frt):
+    # 30 x 52 x 384: 42 pixel-tile pairs x 2 tiles of 192 channels = 42 pair tiles of 18
+    # halos; whole tiles would leave 34 of 76 SM pairs idle, split gives each pair
+    # 756 / 76 = 9.9 halos
+    assert frt.conv_plan(384, 384, 3, 3, 3, 30, 52, 3, sms=152) == \
+        dict(bn=192, pair=1, units=76, split=1, n_tiles=42, nhalo=18)
+    # 60 x 104 x 192: 78 pair tiles on 76 pairs would take two rounds of 9 halos
+    assert frt.conv_plan(192, 192, 3, 3, 3, 60, 104, 3, sms=152) == \
+        dict(bn=192, pair=1, units=76, split=1, n_tiles=78, nhalo=9)
+    # whole tiles only: one round of 126 single-CTA tiles of 128 channels
+    assert frt.conv_plan(384, 384, 3, 3, 3, 30, 52, 3, sms=152, split_mode=1) == \
+        dict(bn=128, pair=0, units=126, split=0, n_tiles=126, nhalo=18)
+    # tiles that fill the units evenly are never split
+    p = frt.conv_plan(384, 384, 3, 3, 3, 30, 52, 3, sms=126, bn=128, pair=0)
+    assert p["split"] == 0 and p["units"] == 126
+    # a forced split of a 2-tile problem: 6 halo steps, at least 2 per unit, so 3 units
+    assert frt.conv_plan(64, 256, 3, 3, 3, 9, 17, 1, sms=152, bn=256, pair=1, split_mode=2,
+                         units=5) == dict(bn=256, pair=1, units=3, split=1, n_tiles=2, nhalo=3)
+    # every plan leaves a tile at most three parts
+    for args in [(384, 384, 3, 3, 3, 30, 52, 3), (192, 192, 3, 3, 3, 60, 104, 3),
+                 (128, 64, 2, 7, 7, 19, 13, 2), (64, 128, 3, 3, 3, 5, 7, 3)]:
+        for sms in (152, 148, 7, 3):
+            p = frt.conv_plan(*args, sms=sms, split_mode=2)
+            if p["split"]:
+                assert p["units"] <= p["n_tiles"] * p["nhalo"] // ((p["nhalo"] + 1) // 2)
+
+
+def test_conv_plan_checks_arguments(frt):
+    with pytest.raises(frt.FrtError):
+        frt.conv_plan(48, 64, 3, 3, 3, 8, 8, 2, sms=152)      # Cin not a multiple of 64
+    with pytest.raises(frt.FrtError):
+        frt.conv_plan(64, 64, 3, 3, 3, 8, 8, 2, sms=152, split_mode=3)

@@ -1,7 +1,8 @@
 """GPU parity of the streaming causal 3D convolution (frt_conv_step) against the fp64
 oracle, through the C ABI: every output element at small sizes (ragged against the
 16-row x 8-column pixel tiles and their halos), every tile width and pairing the kernel
-offers, sampled outputs at the VAE-decoder sizes, the frame cache bit-exact,
+offers, tiles whose K sum is split over several units (parts added by the last to
+arrive), sampled outputs at the VAE-decoder sizes, the frame cache bit-exact,
 determinism and the bf16 output.
 
 Tolerance: fp32 accumulation of K = taps * Cin bf16 products, whatever the order, is
@@ -60,13 +61,15 @@ def test_conv_stream_matches_oracle_every_element(frt, name, out):
     _stream_against_oracle(frt, SMALL[name], name, out)
 
 
-def _stream_against_oracle(frt, cw, name, out, tile=None):
+def _stream_against_oracle(frt, cw, name, out, tile=None, split=None):
     w, b = synth.conv_weights(cw)
     wd, bd = w.cuda(), b.cuda()
     st = frt.ConvStream(cw.cin, cw.cout, cw.kt, cw.kh, cw.kw, cw.grid_h, cw.grid_w, cw.frames,
                         out_dtype=out)
     if tile is not None:
         st.set_tile(*tile)
+    if split is not None:
+        st.set_split(*split)
     outs = []
     orc = OracleConvStream(cw.cin, cw.cout, cw.kt, cw.kh, cw.kw, cw.grid_h, cw.grid_w)
     wf, bf = synth.as_f64(w), b.double().numpy()
@@ -101,10 +104,57 @@ def test_conv_every_tile_matches_oracle(frt, name, bn, pair):
                            tile=(bn, pair))
 
 
+# tiles split over units (forced): the number of units sets where the parts begin, so
+# several counts cover parts of one, two and several halos, a unit holding parts of two
+# tiles, and (pairs) both CTAs of a pair adding their own rows
+SPLIT = [("conv_f1", 128, 0, 5), ("conv_f1", 256, 1, 5), ("conv_f1", 64, 0, 7),
+         ("conv_ragged", 64, 0, 7), ("conv_ragged", 64, 1, 4), ("conv_k7", 64, 1, 3),
+         ("conv_k7", 64, 0, 11), ("conv_odd_tiles", 128, 1, 0), ("conv_f1", 0, 0, 0),
+         ("convtiny", 0, 0, 0)]
+
+
+@pytest.mark.parametrize("name,bn,pair,units", SPLIT)
+@pytest.mark.parametrize("out", [torch.float32, torch.bfloat16])
+def test_conv_split_tiles_match_oracle_every_element(frt, name, bn, pair, units, out):
+    if out == torch.bfloat16 and bn % 64:
+        pytest.skip("bf16 output needs 64-channel units")
+    cw = SMALL[name]
+    plan = frt.conv_plan(cw.cin, cw.cout, cw.kt, cw.kh, cw.kw, cw.grid_h, cw.grid_w, cw.frames,
+                         torch.cuda.get_device_properties(0).multi_processor_count, out_dtype=out,
+                         bn=bn, pair=pair, split_mode=2, units=units)
+    assert plan["split"] == 1, plan
+    _stream_against_oracle(frt, cw, f"{name} bn={bn} pair={pair} units={units}", out,
+                           tile=(bn, pair) if bn else None, split=(2, units))
+
+
+def test_conv_split_is_deterministic(frt):
+    """Parts are added in step order by whichever part arrives last: the same plan gives
+    the same bits on every run."""
+    cw = SMALL["conv_k7"]
+    w, b = (t.cuda() for t in synth.conv_weights(cw))
+    runs = []
+    for _ in range(3):
+        st = frt.ConvStream(cw.cin, cw.cout, cw.kt, cw.kh, cw.kw, cw.grid_h, cw.grid_w, cw.frames)
+        st.set_tile(64, 0)
+        st.set_split(2, 11)
+        ys = []
+        for c in range(cw.chunks):
+            y = st.new_out()
+            st.step(synth.conv_chunk(cw, 2, c).cuda(), w, b, y)
+            ys.append(y)
+        st.sync()
+        st.close()
+        runs.append(ys)
+    for other in runs[1:]:
+        for a, r in zip(runs[0], other):
+            assert torch.equal(a, r)
+
+
 @pytest.mark.parametrize("name", ["conv_f1", "conv_kt1"])
 def test_conv_tile_choice_does_not_change_results(frt, name):
-    """Each output sums the same products in the same order (temporal tap, channel block,
-    spatial tap, 16-channel step) whatever the tile: every choice gives the same bits."""
+    """With whole tiles each output sums the same products in the same order (temporal
+    tap, channel block, spatial tap, 16-channel step) whatever the tile: every choice
+    gives the same bits."""
     cw = SMALL[name]
     w, b = (t.cuda() for t in synth.conv_weights(cw))
     results = {}
@@ -115,6 +165,7 @@ def test_conv_tile_choice_does_not_change_results(frt, name):
             st = frt.ConvStream(cw.cin, cw.cout, cw.kt, cw.kh, cw.kw, cw.grid_h, cw.grid_w,
                                 cw.frames)
             st.set_tile(bn, pr)
+            st.set_split(1)
             ys = []
             for c in range(cw.chunks):
                 y = st.new_out()
@@ -197,6 +248,9 @@ def test_conv_rejects_bad_arguments(frt):
     for bn, pr in ((100, 1), (128, 0), (64, 2)):    # not a width / not dividing Cout / pairing
         with pytest.raises(frt.FrtError):
             st.set_tile(bn, pr)
+    for mode, units in ((3, 0), (-1, 0), (2, -1)):
+        with pytest.raises(frt.FrtError):
+            st.set_split(mode, units)
     st.close()
     # a bf16 output is staged in 64-channel units: a 96-wide tile cannot write it
     cw = SMALL["conv_kt1"]
