@@ -62,6 +62,21 @@ def load_peaks():
         return 1900.0, 6800.0, "fallback"
 
 
+def sustained_tf():
+    """The measured sustained bf16 rate (a GEMM loop held for seconds under the power
+    cap), or None."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops_sustained"])
+    except Exception:
+        return None
+
+
+def of_sustained(achieved: float):
+    sus = sustained_tf()
+    return round(achieved / sus, 4) if sus else None
+
+
 def traffic_record(kernel_file: str, workload: str):
     """DRAM bytes per launch from a committed ncu summary, only if the kernel source is
     unchanged since the capture (sha256 of the .cu file recorded with the counters)."""
@@ -272,6 +287,7 @@ def run_gpu(args, wl, world, rank, local):
                    "attn_flops_per_step": flops},
         "roofline": {"bound": "tensor", "achieved": round(achieved, 2), "peak": peak_tf,
                      "unit": "TFLOP/s", "frac": round(achieved / peak_tf, 4),
+                     "frac_of_sustained": of_sustained(achieved),
                      "traffic": traffic, "kernel": "attn_kernel<128,1,true>",
                      "peak_kind": f"{peak_kind} bf16 dense burst",
                      "launch_ms": round(attn_mean, 4)},
@@ -403,7 +419,8 @@ def run_gpu_multi(args, wl, world, rank, local, dev, peak_tf, peak_kind):
         "config": {"workload": describe(wl) + f", fills {fills} (window = fill per stream)",
                    "note": "step re-rotates the same two input sets in place; timing only"},
         "roofline": {"bound": "tensor", "achieved": round(achieved, 2), "peak": peak_tf,
-                     "unit": "TFLOP/s", "frac": round(achieved / peak_tf, 4), "traffic": None,
+                     "unit": "TFLOP/s", "frac": round(achieved / peak_tf, 4),
+                     "frac_of_sustained": of_sustained(achieved), "traffic": None,
                      "kernel": "attn_kernel<128,32,false>", "peak_kind": peak_kind,
                      "launch_ms": round(attn_mean, 4)},
         "clocks": clk.summary(),
@@ -629,7 +646,8 @@ def run_gpu_block(args, wl, world, rank, local, dev, peak_tf, peak_kind):
                                       "out_projection": out_flops}},
         "roofline": {"bound": "tensor", "achieved": round(tf(attn_flops, attn_ms), 2),
                      "peak": peak_tf, "unit": "TFLOP/s",
-                     "frac": round(tf(attn_flops, attn_ms) / peak_tf, 4), "traffic": None,
+                     "frac": round(tf(attn_flops, attn_ms) / peak_tf, 4),
+                     "frac_of_sustained": of_sustained(tf(attn_flops, attn_ms)), "traffic": None,
                      "kernel": "attn_kernel<128,1,false>", "peak_kind": peak_kind,
                      "launch_ms": round(attn_ms, 4)},
         "projections": {
