@@ -104,6 +104,8 @@ struct ConvParams {
     // arrives last at counters[t * pair + rank] adds all parts in step order
     float4* part;
     int* counters;               // zero between launches: the adding part resets it
+    long long part_cap;          // float4s in part, entries in counters (the FRT_DEBUG
+    long long ctr_cap;           // build checks every derived index against them)
 };
 
 template <int BN, bool PAIR>
@@ -570,6 +572,25 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
                 if (est) report(p.status, abort, 5, it.t);
                 break;
             }
+#ifdef FRT_DEBUG
+            // every workspace row and counter a split tile touches lies inside the
+            // allocations; a tile that fails records FRT_ERR_BOUNDS and the epilogue
+            // stops (the abort flag ends the other roles' waits)
+            if (split) {
+                bool bad = n_parts < 2 || kpart < 0 || kpart >= n_parts ||
+                           (long long)(it.t + 1) * CM > p.ctr_cap;
+                for (int k = 0; k < n_parts && !bad; ++k)
+                    bad = (long long)(part_slot(p, first + k, ts, units, nhalo) * CM + rank + 1) *
+                              (BN / 4) * kBM > p.part_cap;
+                if (bad) {
+                    if (est) {
+                        *abort = 1;
+                        record_status(p.status, kStatusBounds, 307, it.t);
+                    }
+                    break;
+                }
+            }
+#endif
             auto part_row = [&](int k) {                     // this thread's row of part k
                 return p.part + (size_t(part_slot(p, first + k, ts, units, nhalo)) * CM + rank) *
                                     (BN / 4) * kBM + row;
@@ -1215,6 +1236,8 @@ frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w, const void
             return cfail(FRT_ERR_STATE, "split workspace missing: configure the conv again");
         p.part = static_cast<float4*>(c->part);
         p.counters = c->counters;
+        p.part_cap = (long long)(c->part_bytes / sizeof(float4));
+        p.ctr_cap = (long long)c->n_counters;
     }
     const cuuint32_t abox[4] = {64, cuuint32_t(p.halo_w), cuuint32_t(p.halo_h), 1};
     const cuuint64_t xdims[4] = {cuuint64_t(c->cin), cuuint64_t(c->W), cuuint64_t(c->H),
