@@ -47,6 +47,15 @@ int frt_selftest_umma_pair_pv(const void* a, const void* b, float* c, unsigned* 
  * 0, or -1 for another value. */
 int frt_selftest_gemm_force_bn(int bn);
 
+/* How the convolution kernel's split tiles gather their parts in every later
+ * frt_conv_step: 0 as built; 1 without the watch while the first part's MMAs run (the
+ * other parts come only afterwards, by bulk copies into the idle rings); 2 with neither
+ * the watch nor the wait afterwards (the first part writes itself and arrives, and the
+ * part that completes the count adds them all). Every mode gives the same result.
+ * Process-wide and not thread-safe: for tests that cover each path. Returns 0, or -1
+ * for another value. */
+int frt_selftest_conv_part_mode(int mode);
+
 /* Launch a kernel whose one waiting thread waits on an mbarrier that nothing arrives
  * on, bounded by limit_ns (<= 100 ms); it must record FRT_ERR_TIMEOUT in s's status
  * block, which frt_stream_sync then returns. s must be configured. */

@@ -106,6 +106,7 @@ struct ConvParams {
     int* counters;               // zero between launches: the adding part resets it
     long long part_cap;          // float4s in part, entries in counters (the FRT_DEBUG
     long long ctr_cap;           // build checks every derived index against them)
+    int part_mode;               // 0 as built; 1 no watch; 2 no watch, no wait (self-test)
 };
 
 template <int BN, bool PAIR>
@@ -632,7 +633,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
                 }
                 loaded |= fresh;
             };
-            if (split && kpart == 0) {
+            if (split && kpart == 0 && p.part_mode == 0) {
                 const uint64_t t0 = globaltimer_ns();
                 for (;;) {
                     if (est) {
@@ -659,7 +660,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
             }
             tc_fence_after();
             bool early_ready = false;
-            if (split && kpart == 0) {
+            if (split && kpart == 0 && p.part_mode != 2) {
                 // Part 0, accumulator ready: the parts still missing are usually a few
                 // microseconds from arriving (a unit whose whole share lies inside this tile
                 // ends when this one does). Give them kPartWaitNs, taking each as it lands;
@@ -953,6 +954,8 @@ bool plan_rings(int a_bytes, int b_bytes, int kw, int& tb, int& a_stages, int& b
     b_stages = std::min(kMaxStages, (room - a_stages * a_bytes) / (tb * b_bytes));
     return b_stages >= 2;
 }
+
+int g_conv_part_mode = 0;   // self-test override (frt_selftest_conv_part_mode)
 
 // Launch plan of one chunk: tile width, pairing, rings, units and whether tiles are split.
 struct ConvPlan {
@@ -1259,6 +1262,7 @@ frt_status frt_conv_step(frt_conv_t* c, const void* x, const void* w, const void
     p.y_bf16 = c->out_dtype == FRT_OUT_BF16;
     p.wait_limit_ns = c->wait_limit_ns;
     p.status = c->status_dev;
+    p.part_mode = g_conv_part_mode;
     if (c->kt > 1) {
         p.shift_cache = static_cast<const uint4*>(c->cache[c->cur]);
         p.shift_x = static_cast<const uint4*>(x);
@@ -1318,6 +1322,12 @@ frt_status frt_conv_plan(int cin, int cout, int kt, int kh, int kw, int grid_h, 
     plan[4] = pl.n_tiles;
     plan[5] = kt * (cin / kBK);
     return FRT_OK;
+}
+
+int frt_selftest_conv_part_mode(int mode) {
+    if (mode < 0 || mode > 2) return -1;
+    g_conv_part_mode = mode;
+    return 0;
 }
 
 frt_status frt_conv_set_split(frt_conv_t* c, int mode, int units) {

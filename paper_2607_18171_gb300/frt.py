@@ -102,6 +102,7 @@ def lib() -> ctypes.CDLL:
         "frt_selftest_umma_pair": (I, [P, P, P, P, P, P]),
         "frt_selftest_umma_pair_pv": (I, [P, P, P, P, P, P]),
         "frt_selftest_gemm_force_bn": (I, [I]),
+        "frt_selftest_conv_part_mode": (I, [I]),
         "frt_steps_create": (P, [I, I, I, I, I, I]),
         "frt_steps_configure": (I, [P, ctypes.POINTER(Config)]),
         "frt_steps_stream": (P, [P, I]),
@@ -474,6 +475,13 @@ def selftest_gemm_force_bn(bn: int) -> None:
     """Force the projection kernel's tile width (128, 192 or 256; 0 = automatic)."""
     if lib().frt_selftest_gemm_force_bn(bn) != 0:
         raise ValueError("bn must be 0, 128, 192 or 256")
+
+
+def selftest_conv_part_mode(mode: int) -> None:
+    """How split convolution tiles gather their parts (0 as built, 1 no watch, 2 no
+    watch and no wait: the first part writes itself and arrives)."""
+    if lib().frt_selftest_conv_part_mode(mode) != 0:
+        raise ValueError("mode must be 0, 1 or 2")
 
 
 def gemm_plan(M: int, N: int, qkv: bool = False, d: int = 0) -> tuple[int, int]:

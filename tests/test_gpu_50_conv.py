@@ -127,6 +127,30 @@ def test_conv_split_tiles_match_oracle_every_element(frt, name, bn, pair, units,
                            tile=(bn, pair) if bn else None, split=(2, units))
 
 
+@pytest.mark.parametrize("mode", [1, 2])
+@pytest.mark.parametrize("name,bn,pair,units", [SPLIT[0], SPLIT[1], SPLIT[4], SPLIT[6],
+                                                SPLIT[7], SPLIT[9]])
+def test_conv_split_tiles_every_gathering_path(frt, name, bn, pair, units, mode):
+    """The first part of a split tile gathers the others while its MMAs run when they are
+    early; the other paths are forced here: 1 takes every other part only after its own
+    accumulator is ready (bulk copies into the idle rings), 2 makes it write itself and
+    arrive so that whichever part completes the count adds them all. Both match the
+    oracle, and give the bits of the path as built."""
+    cw = SMALL[name]
+    tile = (bn, pair) if bn else None
+    frt.selftest_conv_part_mode(0)
+    base = _stream_against_oracle(frt, cw, f"{name} mode 0", torch.float32, tile=tile,
+                                  split=(2, units))
+    try:
+        frt.selftest_conv_part_mode(mode)
+        got = _stream_against_oracle(frt, cw, f"{name} mode {mode}", torch.float32, tile=tile,
+                                     split=(2, units))
+    finally:
+        frt.selftest_conv_part_mode(0)
+    for c, (a, b) in enumerate(zip(base, got)):
+        assert torch.equal(a, b), f"{name}: gathering mode {mode} changed chunk {c}"
+
+
 def test_conv_split_is_deterministic(frt):
     """Parts are added in step order by whichever part arrives last: the same plan gives
     the same bits on every run."""
