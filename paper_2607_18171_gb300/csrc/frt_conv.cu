@@ -615,9 +615,10 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
             // word (part k sets bit k): every other part that has arrived is added into the
             // idle buffer at once, so that part 0 adds itself at the end with no round trip
             // through memory. With at most two other parts their sum is the same in either
-            // arrival order (two-operand addition commutes). Nothing waits on another CTA:
-            // the watch ends when this CTA's accumulator is ready, and whatever has not
-            // arrived by then goes the write-and-arrive way below.
+            // arrival order (two-operand addition commutes). The watch ends when this
+            // CTA's accumulator is ready; parts still missing then get a bounded wait
+            // (below), and past it everything goes the write-and-arrive way. No wait here
+            // needs another CTA to be resident to end.
             const int others = (1 << n_parts) - 2;           // bits of parts 1 .. n-1
             int loaded = 0;                                   // parts summed into acc2
             auto take = [&](int fresh) {                      // add newly arrived parts
