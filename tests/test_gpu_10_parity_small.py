@@ -32,7 +32,24 @@ SMALL = {
     "max_row": synth.Workload("max_row", 94, 1, 100, 128, 4, 5, 2, 2, 3, (32, 48, 48)),
     # the smallest chunk: one token (1 x 1 grid, one frame); Nkv 1..3, far below one tile
     "one_token": synth.Workload("one_token", 95, 1, 2, 64, 1, 1, 1, 3, 5, (16, 24, 24)),
+    # mixed work split on 152 SMs: 80 heads x 2 query groups (Nq 280) = 160 groups, 152
+    # run whole and the last 8 are cut into KV parts (the dit1p3b / 720p plan, small)
+    "mixed_split_d128": synth.Workload("mixed_split_d128", 98, 1, 80, 128, 7, 20, 2, 2, 3,
+                                       (32, 48, 48)),
+    # the same at head_dim 64: 160 heads x one 256-row group, window 3
+    "mixed_split_d64": synth.Workload("mixed_split_d64", 99, 1, 160, 64, 8, 16, 2, 3, 4,
+                                      (16, 24, 24)),
 }
+
+
+@pytest.mark.parametrize("name", ["mixed_split_d128", "mixed_split_d64"])
+def test_mixed_split_cases_plan_whole_and_cut_groups(frt, name):
+    """The two cases above keep their purpose: on this GPU, at a full window, some query
+    groups run whole and the rest are cut into KV parts merged on the device."""
+    wl = SMALL[name]
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    n_full, n_split = frt.attention_plan([wl.n_q], [wl.window * wl.n_q], wl.heads, sms)
+    assert n_full > 0 and n_split > 1, (n_full, n_split)
 
 
 @pytest.mark.parametrize("name", ["tiny"] + list(SMALL))
