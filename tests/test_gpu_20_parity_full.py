@@ -20,8 +20,10 @@ def frt():
     return m
 
 
+# 720p: chunk 5 is the first full window, chunk 6 the first that evicts (ring slot 0 is
+# rewritten while slots 1-5 keep their chunks)
 @pytest.mark.parametrize("name,check", [("dit1p3b", [6]), ("dit14b", [0, 6, 19]),
-                                        ("stream720p", [5])])
+                                        ("stream720p", [5, 6])])
 def test_full_size_sampled_rows(frt, name, check):
     wl = synth.WORKLOADS[name]
     n_chunks = max(check) + 1
