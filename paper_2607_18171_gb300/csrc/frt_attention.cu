@@ -375,29 +375,33 @@ attn_kernel(const __grid_constant__ AttnParams<MAXS> p) {
         const float sl2 = p.scale_log2;
         bool ok = active;
         if (active) {
-            ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&bars->q_full), 0, lim, abort));
-            if (!ok) report(p.status, abort, 2 + g, -1);
-            if (ROPE && ok && grow < sd.n_q) {
+            // RoPE-Q: every (cos, sin) of the row is loaded first, while the Q tile's TMA
+            // load is still in flight, then the rotation runs once Q has landed. Each
+            // entry is one load from an address chosen without branching (the t segment
+            // lives in the launch parameters, the h and w segments in the stream's
+            // table), so all of them are in flight together; a branch per entry on the
+            // runtime segment widths serialises one load latency per entry.
+            const bool rot = ROPE && grow < sd.n_q;
+            float2 cs[ROPE ? D / 2 : 1];
+            if (rot) {
                 const int f = grow / p.rope.tpf;
                 const int rem = grow - f * p.rope.tpf;
                 const int rr = rem / p.rope.gw;
                 const int col = rem - rr * p.rope.gw;
-                uint8_t* qrow = smem + C::OFF_Q + g * C::Q_TILE + row * 128;
-                // every (cos, sin) of the row first, then the rotation. Each entry is one
-                // load from an address chosen without branching (the t segment lives in
-                // the launch parameters, the h and w segments in the stream's table), so
-                // all of them are in flight together; a branch per entry on the runtime
-                // segment widths serialises one load latency per entry.
-                float2 cs[D / 2];
                 const int dt2 = p.rope.dt2, dth = p.rope.dt2 + p.rope.dh2;
                 const float2* t_row = p.rope.t_tab + f * dt2;
                 const float2* h_row = p.rope.hw + rr * p.rope.dh2 - dt2;
                 const float2* w_row = p.rope.hw + p.rope.gh * p.rope.dh2 + col * p.rope.dw2 - dth;
 #pragma unroll
-                for (int i = 0; i < D / 2; ++i) {
+                for (int i = 0; i < (ROPE ? D / 2 : 0); ++i) {
                     const float2* src = i < dt2 ? t_row + i : (i < dth ? h_row + i : w_row + i);
                     cs[i] = *src;
                 }
+            }
+            ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&bars->q_full), 0, lim, abort));
+            if (!ok) report(p.status, abort, 2 + g, -1);
+            if (ROPE && ok && rot) {
+                uint8_t* qrow = smem + C::OFF_Q + g * C::Q_TILE + row * 128;
 #pragma unroll
                 for (int c = 0; c < D / 8; ++c) {
                     const int cb = c >> 3, cc = c & 7;
