@@ -43,7 +43,6 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
-// Non-blocking test of phase `parity` of an mbarrier (returns at once).
 // atomicAdd with acquire-release semantics at GPU scope. After a barrier of the
 // threads whose writes it publishes, one thread's release makes those writes visible to
 // whoever acquires the new value (release is cumulative over the barrier).
@@ -58,6 +57,7 @@ __device__ __forceinline__ int ld_acquire_gpu(const int* p) {
     asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
 }
+// Non-blocking test of phase `parity` of an mbarrier (returns at once).
 __device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
