@@ -144,6 +144,29 @@ class ClockSampler:
                 "samples": len(sm), "reasons": sorted(reasons)}
 
 
+def clocks_of(clk, step, local, first):
+    """The timed region's clock samples, or, when it was shorter than the sampling
+    interval, samples of the same step run back to back for 0.4 s right after it
+    (labelled as such; the timed numbers are not taken from that run)."""
+    summ = clk.summary()
+    if summ["samples"] > 0:
+        return summ
+    import torch
+    torch.cuda.synchronize()
+    i = first
+    with ClockSampler(local) as probe:
+        t = time.perf_counter()
+        while time.perf_counter() - t < 0.4:
+            for _ in range(20):
+                step(i)
+                i += 1
+            torch.cuda.synchronize()
+    summ = probe.summary()
+    summ["probe"] = ("the same step run back to back for 0.4 s right after the timed region, "
+                     "which is shorter than the sampling interval")
+    return summ
+
+
 def timing_events(n, stream):
     """n (start, stop) CUDA event pairs, recorded once so that the driver-level events
     exist before their handles are handed to the library."""
@@ -531,6 +554,7 @@ def run_gpu_conv(args, cw, world, rank, local):
     st.sync()
     elapsed = max_over_ranks(t0.elapsed_time(t1), world, dev)
     step_ms = statistics.mean(a.elapsed_time(b_) for a, b_ in ev)
+    clocks = clocks_of(clk, step, local, args.warmup + n)
     st.close()
     if world > 1:
         torch.distributed.destroy_process_group()
@@ -552,7 +576,7 @@ def run_gpu_conv(args, cw, world, rank, local):
                      "frac": round(flops / (step_ms * 1e-3) / 1e12 / peak_tf, 4), "traffic": None,
                      "kernel": "conv_kernel (cache update fused)", "peak_kind": peak_kind,
                      "launch_ms": round(step_ms, 4)},
-        "clocks": clk.summary(),
+        "clocks": clocks,
         "gpu_launches": n,
     }
 
@@ -621,6 +645,7 @@ def run_gpu_block(args, wl, world, rank, local, dev, peak_tf, peak_kind):
     attn_ms = statistics.mean(a.elapsed_time(b) for a, b in ev_a)
     qkv_ms = statistics.mean(a.elapsed_time(b) for a, b in ev_q)
     out_ms = statistics.mean(a.elapsed_time(b) for a, b in ev_o)
+    clocks = clocks_of(clk, step, local, args.warmup + n)
     st.close()
     if world > 1:
         torch.distributed.destroy_process_group()
@@ -660,7 +685,7 @@ def run_gpu_block(args, wl, world, rank, local, dev, peak_tf, peak_kind):
                     "frac": round(tf(out_flops, out_ms) / peak_tf, 4)},
             "unit": "TFLOP/s", "peak": peak_tf},
         "attention_share_of_step": round(attn_ms / step_ms, 4),
-        "clocks": clk.summary(),
+        "clocks": clocks,
         "gpu_launches": 3 * n,
     }
 
