@@ -202,6 +202,9 @@ constexpr bool kDebugBuild = false;
 constexpr bool kSlackChunk = false;
 #endif
 
+// staging sets of the host-buffer step (frt_chunk_step_host)
+constexpr int kStageSets = 3;
+
 }  // namespace
 
 struct frt_stream {
@@ -227,12 +230,12 @@ struct frt_stream {
     const void* last_v = nullptr;
     void* stage = nullptr;      // host-API staging: two sets of q, k, v (bf16) and out
     size_t stage_bytes = 0;
-    int stage_turn = 0;         // staging set of the next host-buffer step
+    int stage_turn = 0;         // staging set of the next host-buffer step (of kStageSets)
     cudaStream_t cp_in = nullptr;   // host-to-device copies of host-buffer steps
     cudaStream_t cp_out = nullptr;  // device-to-host copies of host-buffer steps
-    cudaEvent_t ev_in[2] = {nullptr, nullptr};    // inputs of set b landed
-    cudaEvent_t ev_done[2] = {nullptr, nullptr};  // kernels reading set b finished
-    cudaEvent_t ev_out[2] = {nullptr, nullptr};   // output of set b copied out
+    cudaEvent_t ev_in[kStageSets] = {};    // inputs of set b landed
+    cudaEvent_t ev_done[kStageSets] = {};  // kernels reading set b finished
+    cudaEvent_t ev_out[kStageSets] = {};   // output of set b copied out
     unsigned long long wait_limit_ns = kDefaultWaitLimitNs;
     cudaEvent_t ev = nullptr;   // cross-stream ordering for batched launches
     cudaEvent_t attn_start = nullptr;  // caller-owned instrumentation events
@@ -458,7 +461,7 @@ void free_device(frt_stream_t* s) {
     s->ev = nullptr;
     if (s->cp_in) cudaStreamSynchronize(s->cp_in);
     if (s->cp_out) cudaStreamSynchronize(s->cp_out);
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < kStageSets; ++b) {
         if (s->ev_in[b]) cudaEventDestroy(s->ev_in[b]);
         if (s->ev_done[b]) cudaEventDestroy(s->ev_done[b]);
         if (s->ev_out[b]) cudaEventDestroy(s->ev_out[b]);
@@ -872,11 +875,14 @@ frt_status frt_chunk_step_host(frt_stream_t* s, const void* q_host, const void* 
     if (!q_host || !k_host || !v_host || !out_host)
         return fail(FRT_ERR_INVALID_ARG, "NULL host buffer");
     if (s->phase == kRoped) return fail(FRT_ERR_STATE, "a separate rope is pending");
-    // Pipelined: two staging sets alternate; the host-to-device copies of this call run
-    // on a copy stream while the previous call's kernels still run, the device-to-host
-    // copy on a third stream while the next call computes. Events order each set's
-    // reuse: copy-in(n) after compute(n-2), compute(n) after copy-in(n) and after
-    // copy-out(n-2), copy-out(n) after compute(n).
+    // Pipelined: kStageSets staging sets are used in turn; the host-to-device copies of
+    // this call run on a copy stream while earlier calls' kernels still run, the
+    // device-to-host copy on a third stream while later calls compute. Events order each
+    // set's reuse: copy-in(n) after compute(n-S), compute(n) after copy-in(n) and after
+    // copy-out(n-S), copy-out(n) after compute(n) (S = kStageSets). With three sets a
+    // copy may take two kernel steps before compute waits for it: host-device copies
+    // on a shared machine run at their full rate most of the time, with occasional slow
+    // stretches.
     const size_t in_bytes = s->chunk_elems * 2;
     const size_t out_bytes = s->chunk_elems * (s->cfg.out_dtype == FRT_OUT_BF16 ? 2 : 4);
     const size_t per_set = 3 * in_bytes + out_bytes;
@@ -885,22 +891,22 @@ frt_status frt_chunk_step_host(frt_stream_t* s, const void* q_host, const void* 
         if ((e = cudaStreamCreateWithFlags(&s->cp_in, cudaStreamNonBlocking)) != cudaSuccess ||
             (e = cudaStreamCreateWithFlags(&s->cp_out, cudaStreamNonBlocking)) != cudaSuccess)
             return cuda_fail(e, "copy stream creation");
-        for (int b = 0; b < 2; ++b)
+        for (int b = 0; b < kStageSets; ++b)
             if ((e = cudaEventCreateWithFlags(&s->ev_in[b], cudaEventDisableTiming)) != cudaSuccess ||
                 (e = cudaEventCreateWithFlags(&s->ev_done[b], cudaEventDisableTiming)) != cudaSuccess ||
                 (e = cudaEventCreateWithFlags(&s->ev_out[b], cudaEventDisableTiming)) != cudaSuccess)
                 return cuda_fail(e, "event creation");
     }
-    if (s->stage_bytes < 2 * per_set) {
+    if (s->stage_bytes < kStageSets * per_set) {
         if (s->stage) {
             if ((e = cudaDeviceSynchronize()) != cudaSuccess) return cuda_fail(e, "sync");
             cudaFree(s->stage);
             s->stage = nullptr;
             s->stage_bytes = 0;
         }
-        if ((e = cudaMalloc(&s->stage, 2 * per_set)) != cudaSuccess)
+        if ((e = cudaMalloc(&s->stage, kStageSets * per_set)) != cudaSuccess)
             return cuda_fail(e, "staging");
-        s->stage_bytes = 2 * per_set;
+        s->stage_bytes = kStageSets * per_set;
     }
     const int b = s->stage_turn;
     uint8_t* base = static_cast<uint8_t*>(s->stage) + size_t(b) * per_set;
@@ -923,7 +929,7 @@ frt_status frt_chunk_step_host(frt_stream_t* s, const void* q_host, const void* 
             cudaSuccess ||
         (e = cudaEventRecord(s->ev_out[b], s->cp_out)) != cudaSuccess)
         return cuda_fail(e, "device-to-host copy");
-    s->stage_turn ^= 1;
+    s->stage_turn = (s->stage_turn + 1) % kStageSets;
     return FRT_OK;
 }
 
