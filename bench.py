@@ -77,15 +77,25 @@ def of_sustained(achieved: float):
     return round(achieved / sus, 4) if sus else None
 
 
+KERNEL_HEADERS = ("frt_ptx.cuh", "frt_internal.h")
+
+
+def kernel_sources_sha(kernel_file: str) -> str:
+    """sha256 over the kernel's .cu file and the headers it includes, in that order."""
+    h = hashlib.sha256()
+    for name in (kernel_file, *KERNEL_HEADERS):
+        with open(os.path.join(ROOT, "paper_2607_18171_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
 def traffic_record(kernel_file: str, workload: str):
-    """DRAM bytes per launch from a committed ncu summary, only if the kernel source is
-    unchanged since the capture (sha256 of the .cu file recorded with the counters)."""
+    """DRAM bytes per launch from a committed ncu summary, only if the kernel's sources
+    are unchanged since the capture (their sha256, recorded with the counters)."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
-    src = os.path.join(ROOT, "paper_2607_18171_gb300", "csrc", kernel_file)
     try:
         rec = json.load(open(path)).get(workload)
-        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()
-        if rec and rec.get("source_sha256") == sha:
+        if rec and rec.get("sources_sha256") == kernel_sources_sha(kernel_file):
             return rec.get("dram_bytes_per_launch")
     except Exception:
         pass
