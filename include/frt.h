@@ -134,12 +134,12 @@ frt_status frt_chunk_step(frt_stream_t* s, const void* q, const void* k,
 
 /* frt_chunk_step with HOST buffers: copies q, k, v host -> device into
  * stream-owned staging buffers, runs the fused step, copies out device ->
- * host. Consecutive calls are pipelined: two staging sets alternate, the copies
- * in run on an internal copy stream while the previous call's kernels run, and
- * the copy out on another while the next call computes (events keep every set's
+ * host. Consecutive calls are pipelined: three staging sets are used in turn,
+ * the copies in run on an internal copy stream while earlier calls' kernels run,
+ * and the copy out on another while later calls compute (events keep every set's
  * reuse ordered). Host buffers must stay valid, and out_host unread, until
  * frt_stream_sync returns (pinned memory makes the copies asynchronous). The
- * staging (2 x (3 inputs + output)) is allocated on the first call. */
+ * staging (3 x (3 inputs + output)) is allocated on the first call. */
 frt_status frt_chunk_step_host(frt_stream_t* s, const void* q_host,
                                const void* k_host, const void* v_host,
                                void* out_host, int* slot_out,
