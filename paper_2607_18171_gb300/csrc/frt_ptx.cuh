@@ -496,6 +496,8 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
     return r;
 }
+__device__ __forceinline__ float bf16lo_to_f32(uint32_t x) { return __uint_as_float(x << 16); }
+__device__ __forceinline__ float bf16hi_to_f32(uint32_t x) { return __uint_as_float(x & 0xFFFF0000u); }
 
 // Packed fp32 pairs (sm_100+ f32x2 arithmetic): one instruction for two lanes of work.
 __device__ __forceinline__ uint64_t f2_pack(float lo, float hi) {
